@@ -1,0 +1,420 @@
+#!/usr/bin/env python3
+"""Benchmark of batched Traversal Verification (arXiv 2505.12398) on GB300.
+
+One step = one call of the library's verification (tv_verify_batch) over one
+batch of synthetic draft trees whose inputs are resident in HBM: the row
+normalisers of every internal row, the serial leaf-to-root traversal of
+every tree with its vocabulary-wide rejection passes, and the bonus-token
+draw.  L2 is flushed (a 256 MiB write) before every timed step, outside the
+timed interval.  Times are CUDA-event device times on the launching stream.
+
+Prints ONE JSON line (rank 0).  ``--impl reference`` times the CPU oracle
+(the slow literal float64 restatement of the paper's algorithm) on the host
+cores instead, on a bounded sample of the same workload per step.
+"""
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+DEFAULT_WORKLOAD = "eagle_v128k"
+
+
+def parse_args():
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--batch", type=int, default=None)
+    ap.add_argument("--sigma", type=float, default=None)
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0,
+                    help="rough budget of the CPU-baseline sample")
+    return ap.parse_args()
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+# ----------------------------------------------------------- clocks ---------
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu_index = gpu_index
+        self.proc = None
+        self.file = None
+
+    def start(self):
+        try:
+            self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "50", "-i", str(self.gpu_index)],
+                stdout=self.file, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.file.flush()
+        self.file.seek(0)
+        rows = [r.split(",") for r in self.file.read().strip().splitlines() if r.strip()]
+        os.unlink(self.file.name)
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            r = [x.strip() for x in r]
+            if len(r) < 9:
+                continue
+            try:
+                sm.append(float(r[1]))
+                smax = float(r[2])
+            except ValueError:
+                continue
+            for k, name in enumerate(names):
+                if r[5 + k].lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": smax,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------- CPU oracle ---------
+
+def dump_sample(inp, trees, tmpdir):
+    """Host copies of a sample of trees (float32 logits) for the oracle."""
+    import numpy as np
+    idx = list(trees)
+    path = os.path.join(tmpdir, "sample.npz")
+    np.savez(path, parents=inp.parents[idx].cpu().numpy(), tokens=inp.tokens[idx].cpu().numpy(),
+             logits=inp.logits[idx].float().cpu().numpy(),
+             drafts=inp.draft_probs[idx].cpu().numpy(), uniforms=inp.uniforms[idx].cpu().numpy())
+    # npz members cannot be memory-mapped; expand to a directory of .npy files
+    d = np.load(path)
+    outdir = os.path.join(tmpdir, "sample")
+    os.makedirs(outdir, exist_ok=True)
+    for k in d.files:
+        np.save(os.path.join(outdir, k + ".npy"), d[k])
+    os.unlink(path)
+    return outdir
+
+
+class _DirArrays:
+    def __init__(self, path):
+        import numpy as np
+        self.d = {k[:-4]: np.load(os.path.join(path, k), mmap_mode="r")
+                  for k in os.listdir(path) if k.endswith(".npy")}
+
+    def __getitem__(self, k):
+        return self.d[k]
+
+
+def _oracle_dir_worker(args):
+    path, b, temperature = args
+    from oracle.verify import verify_tree
+    d = _DirArrays(path)
+    r = verify_tree(d["parents"][b], d["tokens"][b], d["logits"][b], d["drafts"][b],
+                    temperature, d["uniforms"][b])
+    return r["tau"]
+
+
+def time_oracle(sample_dir, n_trees, temperature, pool, reps=1):
+    jobs = [(sample_dir, b % n_trees, temperature) for b in range(n_trees * reps)]
+    t0 = time.perf_counter()
+    pool.map(_oracle_dir_worker, jobs, chunksize=1)
+    return time.perf_counter() - t0, len(jobs)
+
+
+# ---------------------------------------------------------- helpers ---------
+
+def algorithmic_bytes(parents, stats, V, logit_bytes):
+    """Per tree: one target row per internal node, one draft row per node with
+    at least one rejection pass, the accepted leaf's target row (the eager
+    reading of Algorithm 3's initialisation)."""
+    import torch
+    B, R = parents.shape
+    has_child = torch.zeros(B, R, dtype=torch.bool, device=parents.device)
+    p = parents[:, 1:].long()
+    has_child.scatter_(1, p.clamp(min=0), True)
+    n_int = has_child.sum(1).to(torch.int64)
+    rej = stats[:, 2].to(torch.int64)
+    leaf = stats[:, 3].to(torch.int64)
+    row_bytes = n_int * V * logit_bytes
+    other = rej * V * 4 + leaf * V * logit_bytes
+    return int(row_bytes.sum()), int(other.sum())
+
+
+def main():
+    args = parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        return run_reference(args, world, rank)
+
+    import torch
+    import torch.distributed as dist
+    import paper_2505_12398_gb300 as tv
+    from paper_2505_12398_gb300.build import build
+    from workloads.synth import get_workload, make_inputs
+
+    if world > 1:
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local_rank if world > 1 else 0)
+    torch.cuda.set_device(dev)
+    build()
+
+    w = get_workload(args.workload, batch=args.batch, sigma=args.sigma)
+    inp = make_inputs(w, seed=args.seed + 7919 * rank, device=dev)
+    B, R = inp.parents.shape
+    N, V = R - 1, w.vocab
+    lb = 2 if inp.logits.dtype == torch.bfloat16 else 4
+    v = tv.Verifier(V, N, B, "bf16" if lb == 2 else "fp32", device=dev.index)
+    stream = torch.cuda.current_stream(dev)
+
+    # decisions are a deterministic function of the inputs: one instrumented
+    # call gives the rows each tree needs (algorithmic bytes) and tau
+    _, tau_d, _, _, stats = v.verify(inp.parents, inp.tokens, inp.logits, inp.draft_probs,
+                                     inp.temperature, inp.uniforms, debug=True)
+    torch.cuda.synchronize(dev)
+    row_bytes, trav_bytes = algorithmic_bytes(inp.parents, stats, V, lb)
+    a_bytes = row_bytes + trav_bytes
+    mean_tau1 = float(tau_d.float().mean()) + 1.0
+    passes_per_tree = float(stats[:, 1].float().mean())
+
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    out = (torch.empty(B, N, dtype=torch.int32, device=dev),
+           torch.empty(B, dtype=torch.int32, device=dev),
+           torch.empty(B, dtype=torch.int32, device=dev))
+    v.set_phase_timing(True)
+    for _ in range(args.warmup):
+        flush.zero_()
+        v.verify(inp.parents, inp.tokens, inp.logits, inp.draft_probs, inp.temperature,
+                 inp.uniforms, out=out, stream=stream)
+    torch.cuda.synchronize(dev)
+
+    gpu_idx = 0
+    cvd = os.environ.get("CUDA_VISIBLE_DEVICES", "")
+    if cvd and cvd.split(",")[dev.index].strip().isdigit():
+        gpu_idx = int(cvd.split(",")[dev.index])
+    sampler = ClockSampler(gpu_idx)
+    sampler.start()
+    time.sleep(0.3)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    step_ms, phase = [], []
+    e0 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    e1 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    wall0 = time.perf_counter()
+    for k in range(args.steps):
+        flush.zero_()
+        e0[k].record(stream)
+        v.verify(inp.parents, inp.tokens, inp.logits, inp.draft_probs, inp.temperature,
+                 inp.uniforms, out=out, stream=stream)
+        e1[k].record(stream)
+        phase.append(v.last_phase_ms())
+    torch.cuda.synchronize(dev)
+    wall = time.perf_counter() - wall0
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop()
+    step_ms = [e0[k].elapsed_time(e1[k]) for k in range(args.steps)]
+    total_ms = sum(step_ms)
+    t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    total_ms_max = float(t.item())
+    v.set_phase_timing(False)
+
+    # end to end through the public API from pinned host buffers
+    e2e = None
+    if not args.no_e2e:
+        hp = [x.cpu().pin_memory() for x in (inp.parents, inp.tokens, inp.logits,
+                                              inp.draft_probs, inp.uniforms)]
+        hout = (torch.empty(B, N, dtype=torch.int32).pin_memory(),
+                torch.empty(B, dtype=torch.int32).pin_memory(),
+                torch.empty(B, dtype=torch.int32).pin_memory())
+        v.verify_host(hp[0], hp[1], hp[2], hp[3], inp.temperature, hp[4], hout, stream=stream)
+        ks = max(1, args.e2e_steps)
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+        x0 = torch.cuda.Event(enable_timing=True)
+        x1 = torch.cuda.Event(enable_timing=True)
+        x0.record(stream)
+        for _ in range(ks):
+            v.verify_host(hp[0], hp[1], hp[2], hp[3], inp.temperature, hp[4], hout,
+                          stream=stream)
+        x1.record(stream)
+        torch.cuda.synchronize(dev)
+        e_ms = x0.elapsed_time(x1)
+        te = torch.tensor([e_ms], dtype=torch.float64, device=dev)
+        if world > 1:
+            dist.all_reduce(te, op=dist.ReduceOp.MAX)
+        h2d = sum(x.numel() * x.element_size() for x in hp)
+        d2h = sum(x.numel() * x.element_size() for x in hout)
+        assert torch.equal(hout[1], out[1].cpu()), "host entry point disagrees"
+        e2e = {"value": round(B * world * ks / (float(te.item()) / 1e3), 3), "unit": "trees/s",
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": ks}
+
+    # CPU baseline: the oracle on host cores, bounded sample of the same batch
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(inp, args, B)
+
+    peak, peak_kind = measured_peaks()
+    ph = [sum(p[i] for p in phase) / len(phase) for i in range(3)]
+    names = ["tv_prep_kernel", "tv_row_stats_kernel", "tv_traverse_kernel"]
+    kbytes = [0, row_bytes, trav_bytes]
+    dom = max(range(3), key=lambda i: ph[i])
+    ms_step = total_ms_max / args.steps
+    trees_s = B * world * args.steps / (total_ms_max / 1e3)
+    step_gbs = a_bytes / (ms_step / 1e3) / 1e9
+    dom_gbs = kbytes[dom] / (ph[dom] / 1e3) / 1e9 if ph[dom] > 0 else 0.0
+    line = {
+        "metric": "verified trees/sec and logit GB/s (fraction of HBM peak) at batch B, "
+                  "vocab V, 1 GB300",
+        "value": round(trees_s, 3),
+        "unit": "trees/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_step, 6),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f32",
+        "data": "synthetic (seeded logits with Zipf rank prior, noisy-drafter probabilities, "
+                "EAGLE-shaped draft trees sampled without replacement)",
+        "config": {"workload": w.name, "batch": B, "vocab": V, "nodes": N,
+                   "internal_rows": int(row_bytes // (V * lb) // B) if B else 0,
+                   "logit_dtype": "bf16" if lb == 2 else "fp32",
+                   "temperature": w.temperature, "sigma": w.sigma, "seed": args.seed,
+                   "l2": "flushed by a 256 MiB write before every timed step (untimed)",
+                   "parallelism": f"dp{world} (independent trees per GPU)"},
+        "verified_logit_gbps": round(step_gbs, 2),
+        "hbm_frac_step": round(step_gbs / peak, 4),
+        "algorithmic_bytes_per_step": a_bytes,
+        "mean_accept_len_tau_plus_1": round(mean_tau1, 4),
+        "rejection_passes_per_tree": round(passes_per_tree, 3),
+        "phase_ms": {names[i]: round(ph[i], 6) for i in range(3)},
+        "roofline": {"bound": "hbm", "kernel": names[dom], "achieved": round(dom_gbs, 2),
+                     "peak": peak, "unit": "GB/s", "frac": round(dom_gbs / peak, 4),
+                     "peak_kind": peak_kind, "bytes_per_launch": kbytes[dom],
+                     "traffic": None},
+        "roofline_step": {"bound": "hbm", "achieved": round(step_gbs, 2), "peak": peak,
+                          "unit": "GB/s", "frac": round(step_gbs / peak, 4)},
+        "e2e": e2e,
+        "gpu_launches": 3 * args.steps,
+        "clocks": clocks,
+        "cpu_baseline": cpu,
+        "wall_s_timed_region": round(wall, 3),
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    v.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def cpu_baseline(inp, args, B):
+    import multiprocessing as mp
+    cores = os.cpu_count() or 1
+    with tempfile.TemporaryDirectory() as td:
+        n_sample = min(B, max(cores, 8))
+        sdir = dump_sample(inp, range(n_sample), td)
+        ctx = mp.get_context("spawn")
+        with ctx.Pool(cores) as pool:
+            # one probe tree per worker to size the sample to the time budget
+            t_probe, n_probe = time_oracle(sdir, n_sample, inp.temperature, pool)
+            per_round = max(t_probe, 1e-3)
+            reps = max(1, min(50, int(args.cpu_seconds / per_round)))
+            t, n = time_oracle(sdir, n_sample, inp.temperature, pool, reps=reps)
+    return {"value": round(n / t, 4), "unit": "trees/s", "cores": cores, "kind": "oracle",
+            "sample": f"{n} oracle tree verifications ({n_sample} distinct trees of the same "
+                      f"batch, repeated {reps}x) across {cores} spawn workers, {t:.1f} s"}
+
+
+def run_reference(args, world, rank):
+    """The oracle (float64 CPU restatement of Algorithm 3) as the reference arm."""
+    if rank != 0:
+        return
+    import multiprocessing as mp
+    from workloads.synth import get_workload, make_inputs
+    w = get_workload(args.workload, batch=args.batch, sigma=args.sigma)
+    cores = os.cpu_count() or 1
+    per_step = max(1, min(w.batch, cores))
+    # the same workload, drawn on the CPU; only the sampled trees are needed
+    gen_w = get_workload(args.workload, batch=per_step, sigma=args.sigma)
+    inp = make_inputs(gen_w, seed=args.seed, device="cpu")
+    with tempfile.TemporaryDirectory() as td:
+        sdir = dump_sample(inp, range(per_step), td)
+        ctx = mp.get_context("spawn")
+        with ctx.Pool(cores) as pool:
+            for _ in range(args.warmup):
+                time_oracle(sdir, per_step, inp.temperature, pool)
+            times = []
+            for _ in range(args.steps):
+                t, _ = time_oracle(sdir, per_step, inp.temperature, pool)
+                times.append(t)
+    total = sum(times)
+    value = per_step * args.steps / total
+    line = {
+        "impl": "reference",
+        "metric": "verified trees/sec and logit GB/s (fraction of HBM peak) at batch B, "
+                  "vocab V, 1 GB300",
+        "value": round(value, 4), "unit": "trees/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(total / args.steps * 1e3, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": {"workload": w.name, "batch": w.batch, "vocab": w.vocab,
+                                         "nodes": w.nodes},
+        "cpu_baseline": {"value": round(value, 4), "unit": "trees/s", "cores": cores,
+                         "kind": "oracle",
+                         "sample": f"{per_step} trees of the workload per step, one per "
+                                   f"spawn worker"},
+        "e2e": {"value": round(value, 4), "unit": "trees/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,199 @@
+/*
+ * tv.h -- C ABI of the GB300 batched Traversal Verification library.
+ *
+ * Traversal Verification (arXiv 2505.12398, §3.1, Algorithm 3) verifies a
+ * speculative-decoding draft token tree against the target model from the
+ * leaves towards the root and accepts whole root-to-node sequences.  Given a
+ * decoding tree T (Definition 1, §3.3), the draft distributions M_s(.|X^i) of
+ * its non-leaf nodes and the target distributions M_b(.|X^i) of all its
+ * nodes, it returns an accepted chain X^tau and one more token Y whose joint
+ * law is the target model's (Definition 2, Theorem 1).  This library runs
+ * that algorithm for a batch of independent trees on one GPU.
+ *
+ * Conventions shared by every call:
+ *   - B trees, each with N draft nodes plus the root: N+1 rows per tree.
+ *     Row 0 is the root (the prefix X_0); rows 1..N are draft nodes.
+ *   - Every array pointer is a DEVICE pointer owned by the caller (except in
+ *     tv_verify_batch_host).  The library never frees or retains it.
+ *   - Layouts are dense, row-major, with no padding: [B][N+1] for tree
+ *     arrays, [B][N+1][V] for the per-row distributions, [B][N+2] for the
+ *     uniforms.  Distribution arrays must start on a 16-byte boundary.
+ *   - All work is queued on the caller's CUDA stream (a cudaStream_t passed
+ *     as void*; NULL = the legacy default stream).  Calls return as soon as
+ *     the work is queued; nothing in the library synchronises the host
+ *     except tv_get_status and tv_verify_batch_host.
+ *   - Return values: 0 on success, a negative TV_ERR_* code otherwise.  Bad
+ *     arguments are caught on the host before anything is launched.  Bad
+ *     trees are found on the device: that tree's outputs are set to -1 and a
+ *     TV_STATUS_* bit is raised in the handle's status word.
+ *   - A handle owns its device workspace and may serve one stream at a time:
+ *     calls on different streams that may overlap need different handles.
+ */
+#ifndef TV_H_
+#define TV_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct tv_handle tv_handle;
+
+/* Element type of the target logits. */
+typedef enum { TV_BF16 = 0, TV_FP32 = 1 } tv_dtype;
+
+/* Return codes. */
+enum {
+  TV_OK = 0,
+  TV_ERR_INVALID_ARG = -1, /* null pointer, negative size, bad flag, misaligned array */
+  TV_ERR_TEMPERATURE = -2, /* temperature not finite and > 0 (the method samples; §G) */
+  TV_ERR_VOCAB = -3,       /* vocabulary size out of range */
+  TV_ERR_CAPACITY = -4,    /* B or N above what the handle was created for */
+  TV_ERR_CUDA = -5,        /* a CUDA runtime call failed (no device, launch error, ...) */
+  TV_ERR_DEVICE = -6       /* the handle's device is not a supported GPU */
+};
+
+/* Device-side status bits, OR-ed into the handle's status word. */
+enum {
+  TV_STATUS_BAD_TREE = 1u,     /* parents[b][0] != -1 or parents[b][i] not in [0, i) */
+  TV_STATUS_BAD_TOKEN = 2u,    /* a draft token outside [0, V) */
+  TV_STATUS_DUP_SIBLING = 4u,  /* two siblings carry the same token (Definition 1
+                                  draws children without replacement) */
+  TV_STATUS_ZERO_DRAFT = 8u,   /* a drafted token has zero draft probability at its
+                                  parent, so it cannot have come from M_s */
+  TV_STATUS_DEGENERATE = 16u   /* informational: S = 0 occurred in Eqs. (1)/(3); the
+                                  0/0 was resolved as p' = 0 (p < 1) or p' = 1 (p = 1) */
+};
+
+/* Flags for tv_create. */
+enum { TV_FLAG_NONE = 0u };
+
+/*
+ * tv_create -- allocate a handle and its device workspace.
+ *   out        : receives the handle (set to NULL on failure).
+ *   device     : CUDA device ordinal the handle works on.
+ *   vocab      : V, the vocabulary size (1 <= V <= 2^28).
+ *   max_nodes  : largest N (draft nodes per tree, root excluded) later calls
+ *                may pass; 0 <= max_nodes <= 1023.
+ *   max_batch  : largest B later calls may pass; >= 1.
+ *   logit_dtype: element type of target_logits in later calls.
+ *   flags      : TV_FLAG_NONE.
+ * Errors: TV_ERR_INVALID_ARG, TV_ERR_VOCAB, TV_ERR_CUDA, TV_ERR_DEVICE.
+ */
+int tv_create(tv_handle** out, int device, int vocab, int max_nodes, int max_batch,
+              tv_dtype logit_dtype, unsigned flags);
+
+/*
+ * tv_verify_batch -- Traversal Verification of B trees (Algorithm 3, §3.1).
+ *
+ * Inputs (device pointers):
+ *   parents          [B][N+1] int32.  parents[b][0] = -1; for i >= 1 the parent
+ *                    row of node i, with 0 <= parents[b][i] < i.  Children of a
+ *                    node are taken in increasing row order; the traversal
+ *                    visits the tree in post-order (Appendix E).
+ *   draft_tokens     [B][N+1] int32.  Token X_i of node i, 0 <= X_i < V;
+ *                    entry 0 is ignored.  Siblings must carry distinct tokens.
+ *   target_logits    [B][N+1][V], bf16 or fp32 (tv_create's logit_dtype).
+ *                    Row i holds the target model's logits at node i;
+ *                    M_b(.|X^i) = softmax(logits / temperature).  Rows of every
+ *                    node are needed (a leaf's row when it is accepted).
+ *   draft_probs      [B][N+1][V] fp32.  Row i holds M_s(.|X^i), used as given
+ *                    (not renormalised, no temperature applied).  Rows of leaf
+ *                    nodes are never read.
+ *   temperature      > 0; scales the target logits only.
+ *   uniforms         [B][N+2] fp32 in [0, 1).  uniforms[b][i] (1 <= i <= N) is the
+ *                    eta of the test of node i (accepted iff eta < p, strict);
+ *                    uniforms[b][N+1] draws the bonus token Y.  Entry 0 is unused.
+ *                    Each node is tested at most once, so one uniform per node
+ *                    has the law of Algorithm 3's fresh draw per test.
+ * Outputs (device pointers, written for every tree b < B):
+ *   out_accepted_path[B][N]  node ids of the accepted chain X^tau from depth 1
+ *                    to depth tau (the root excluded), then -1 padding.
+ *   out_accept_len   [B] tau, the number of accepted draft tokens (0..N);
+ *                    -1 marks an invalid tree (see TV_STATUS_*).
+ *   out_bonus_token  [B] Y, drawn by inverse CDF (smallest y with
+ *                    u * W < sum_{x<=y} w(x)) from the accepted node's current
+ *                    target distribution: its original M_b for an original
+ *                    leaf, else the residual left by Eqs. (1)-(3); -1 if invalid.
+ *   cuda_stream      cudaStream_t the work is queued on.
+ * Errors (host-side, nothing launched): TV_ERR_INVALID_ARG, TV_ERR_TEMPERATURE,
+ * TV_ERR_CAPACITY; TV_ERR_CUDA if a launch fails.  B = 0 is a no-op.
+ */
+int tv_verify_batch(tv_handle* h, int B, int N, const int32_t* parents,
+                    const int32_t* draft_tokens, const void* target_logits,
+                    const float* draft_probs, float temperature, const float* uniforms,
+                    int32_t* out_accepted_path, int32_t* out_accept_len,
+                    int32_t* out_bonus_token, void* cuda_stream);
+
+/*
+ * tv_verify_batch_debug -- tv_verify_batch plus per-node instrumentation.
+ *   out_node_p  [B][N+1] fp32 (device): the acceptance rate p of node i at the
+ *               moment it was tested (Algorithm 3's eta < p test); 0 for a node
+ *               removed because its rate reached 0 (§3.2); NaN for nodes never
+ *               tested; entry 0 (root) NaN.
+ *   out_stats   [B][4] int32 (device): { number of tests, number of
+ *               S-computations (Eqs. (1)/(3), one vocabulary pass each), number
+ *               of distinct nodes with at least one S-computation, 1 if the
+ *               bonus token came from an original leaf's row else 0 }.
+ * Either pointer may be NULL.  Other arguments and errors as tv_verify_batch.
+ */
+int tv_verify_batch_debug(tv_handle* h, int B, int N, const int32_t* parents,
+                          const int32_t* draft_tokens, const void* target_logits,
+                          const float* draft_probs, float temperature,
+                          const float* uniforms, int32_t* out_accepted_path,
+                          int32_t* out_accept_len, int32_t* out_bonus_token,
+                          float* out_node_p, int32_t* out_stats, void* cuda_stream);
+
+/*
+ * tv_verify_batch_host -- the same verification from HOST buffers: copies the
+ * inputs to device staging owned by the handle (allocated on first use, sized
+ * by tv_create's limits), runs tv_verify_batch on cuda_stream, copies the
+ * three outputs back and synchronises the stream before returning.  All
+ * pointers are host pointers with the layouts above; pinned (page-locked)
+ * memory gives the fastest copies.  Errors as tv_verify_batch.
+ */
+int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
+                         const int32_t* draft_tokens, const void* target_logits,
+                         const float* draft_probs, float temperature,
+                         const float* uniforms, int32_t* out_accepted_path,
+                         int32_t* out_accept_len, int32_t* out_bonus_token,
+                         void* cuda_stream);
+
+/*
+ * tv_get_status -- synchronise the handle's device and return, in *status, the
+ * OR of the TV_STATUS_* bits raised since the previous tv_get_status call
+ * (then clear them).  Errors: TV_ERR_INVALID_ARG, TV_ERR_CUDA.
+ */
+int tv_get_status(tv_handle* h, uint32_t* status);
+
+/*
+ * tv_set_phase_timing -- when enable != 0, later verify calls on this handle
+ * record CUDA events on their stream around each of the three kernels
+ * (row preparation, row normalisers, traversal).  Costs three event records
+ * per call; off by default.  Errors: TV_ERR_INVALID_ARG, TV_ERR_CUDA.
+ */
+int tv_set_phase_timing(tv_handle* h, int enable);
+
+/*
+ * tv_last_phase_ms -- waits for the events of the most recent timed call and
+ * writes the device time of its three kernels, in milliseconds, to ms[0..2]
+ * (preparation, row normalisers, traversal).  Errors: TV_ERR_INVALID_ARG
+ * (timing off or no timed call yet), TV_ERR_CUDA.
+ */
+int tv_last_phase_ms(tv_handle* h, float* ms);
+
+/* tv_destroy -- free the handle's workspace (synchronises its device). */
+int tv_destroy(tv_handle* h);
+
+/* tv_strerror -- static description of a return code. */
+const char* tv_strerror(int code);
+
+/* tv_version -- library version, major * 10000 + minor * 100 + patch. */
+int tv_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TV_H_ */

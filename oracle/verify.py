@@ -46,7 +46,7 @@ def inverse_cdf(w, u):
     return y, float(margin), float(W)
 
 
-def verify_tree(parents, tokens, logits, draft_probs, temperature, uniforms):
+def verify_tree(parents, tokens, logits, draft_probs, temperature, uniforms, keep_cdf=False):
     """Traversal Verification of one tree.
 
     ``logits`` / ``draft_probs`` are [N+1, V] arrays (any float dtype; bf16
@@ -87,6 +87,7 @@ def verify_tree(parents, tokens, logits, draft_probs, temperature, uniforms):
         node_p[c] = 0.0
     w = st.bonus_weights(accepted)
     y, y_margin, W = inverse_cdf(w, u[n])
+    cdf = np.cumsum(np.asarray(w, dtype=np.float64)) if keep_cdf else None
     path = st.path(accepted)
     internal = [i for i in range(n) if st.children[i]]
     return {
@@ -106,6 +107,8 @@ def verify_tree(parents, tokens, logits, draft_probs, temperature, uniforms):
         "leaf_row_read": accepted not in st.mb,
         "pruned": list(st.pruned),
         "degenerate": st.degenerate,
+        "bonus_u": float(u[n]),
+        "bonus_cdf": cdf,
     }
 
 
@@ -120,7 +123,7 @@ def algorithmic_bytes(result, vocab, logit_bytes):
 
 
 def verify_batch(parents, tokens, logits, draft_probs, temperature, uniforms,
-                 trees=None):
+                 trees=None, keep_cdf=False):
     """Batch driver: arrays [B, N+1], [B, N+1], [B, N+1, V], [B, N+1, V],
     scalar, [B, N+2].  Invalid trees get tau = -1, bonus = -1 and an all -1
     path, the same marking the library uses.  ``trees`` restricts the work to a
@@ -135,7 +138,7 @@ def verify_batch(parents, tokens, logits, draft_probs, temperature, uniforms,
     for b in idx:
         try:
             r = verify_tree(parents[b], tokens[b], logits[b], draft_probs[b],
-                            temperature, uniforms[b])
+                            temperature, uniforms[b], keep_cdf=keep_cdf)
         except InvalidTree as e:
             out_tau[b] = -1
             out_bonus[b] = -1

@@ -1,0 +1,205 @@
+"""ctypes binding of libtv.so (C ABI in include/tv.h)."""
+
+import ctypes
+import os
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+
+TV_BF16 = 0
+TV_FP32 = 1
+TV_STATUS = {
+    "BAD_TREE": 1,
+    "BAD_TOKEN": 2,
+    "DUP_SIBLING": 4,
+    "ZERO_DRAFT": 8,
+    "DEGENERATE": 16,
+}
+
+
+class LibraryError(RuntimeError):
+    """A call into libtv.so returned an error code."""
+
+    def __init__(self, fn, code, lib):
+        msg = lib.tv_strerror(code).decode() if lib is not None else "?"
+        super().__init__(f"{fn} failed with code {code}: {msg}")
+        self.code = code
+
+
+def library_path():
+    return os.path.join(HERE, "libtv.so")
+
+
+_LIB = None
+
+_P = ctypes.c_void_p
+_I = ctypes.c_int
+_F = ctypes.c_float
+
+_SIGS = {
+    "tv_create": (_I, [ctypes.POINTER(_P), _I, _I, _I, _I, _I, ctypes.c_uint]),
+    "tv_verify_batch": (_I, [_P, _I, _I, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P]),
+    "tv_verify_batch_debug": (_I, [_P, _I, _I, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P, _P, _P]),
+    "tv_verify_batch_host": (_I, [_P, _I, _I, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P]),
+    "tv_get_status": (_I, [_P, ctypes.POINTER(ctypes.c_uint32)]),
+    "tv_destroy": (_I, [_P]),
+    "tv_set_phase_timing": (_I, [_P, _I]),
+    "tv_last_phase_ms": (_I, [_P, ctypes.POINTER(ctypes.c_float)]),
+    "tv_strerror": (ctypes.c_char_p, [_I]),
+    "tv_version": (_I, []),
+}
+
+
+def library():
+    """Load libtv.so (raises if it has not been built: there is no fallback)."""
+    global _LIB
+    if _LIB is None:
+        path = library_path()
+        if not os.path.exists(path):
+            raise ImportError(
+                f"{path} is missing: build it with `python -m paper_2505_12398_gb300.build` "
+                "(or __graft_entry__.build()); the verifier has no CPU implementation")
+        lib = ctypes.CDLL(path)
+        for name, (res, args) in _SIGS.items():
+            fn = getattr(lib, name)
+            fn.restype = res
+            fn.argtypes = args
+        _LIB = lib
+    return _LIB
+
+
+def status_names(bits):
+    return [k for k, v in TV_STATUS.items() if bits & v]
+
+
+def _ptr(t):
+    return ctypes.c_void_p(t.data_ptr()) if t is not None else ctypes.c_void_p(0)
+
+
+def _stream_ptr(stream):
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+class Verifier:
+    """Owns a ``tv_handle`` (device workspace) for one device and size limits.
+
+    All tensors passed to :meth:`verify` must be contiguous CUDA tensors on
+    the handle's device with the dtypes and layouts of include/tv.h.
+    """
+
+    def __init__(self, vocab, max_nodes, max_batch, logit_dtype="bf16", device=0):
+        import torch
+        self.lib = library()
+        if logit_dtype in ("bf16", torch.bfloat16, TV_BF16):
+            self.dtype_code, self.logit_dtype = TV_BF16, torch.bfloat16
+        elif logit_dtype in ("fp32", torch.float32, TV_FP32):
+            self.dtype_code, self.logit_dtype = TV_FP32, torch.float32
+        else:
+            raise ValueError(f"unsupported logit dtype {logit_dtype}")
+        self.vocab, self.max_nodes, self.max_batch = vocab, max_nodes, max_batch
+        self.device = torch.device("cuda", device) if isinstance(device, int) else torch.device(device)
+        h = ctypes.c_void_p()
+        rc = self.lib.tv_create(ctypes.byref(h), self.device.index or 0, vocab, max_nodes,
+                                max_batch, self.dtype_code, 0)
+        if rc != 0:
+            raise LibraryError("tv_create", rc, self.lib)
+        self.handle = h
+
+    def close(self):
+        if getattr(self, "handle", None) is not None and self.handle.value:
+            self.lib.tv_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def _check(self, parents, tokens, logits, drafts, uniforms):
+        import torch
+        B, R = parents.shape
+        N = R - 1
+        V = self.vocab
+        exp = [(parents, torch.int32, (B, R)), (tokens, torch.int32, (B, R)),
+               (logits, self.logit_dtype, (B, R, V)), (drafts, torch.float32, (B, R, V)),
+               (uniforms, torch.float32, (B, R + 1))]
+        for t, dt, shape in exp:
+            if t.dtype != dt or tuple(t.shape) != shape:
+                raise ValueError(f"expected {dt} {shape}, got {t.dtype} {tuple(t.shape)}")
+            if not t.is_contiguous():
+                raise ValueError("tensors must be contiguous")
+            if t.device != self.device:
+                raise ValueError(f"tensor on {t.device}, handle on {self.device}")
+        return B, N
+
+    def verify(self, parents, tokens, logits, drafts, temperature, uniforms,
+               out=None, stream=None, debug=False):
+        """Returns (path [B,N] int32, tau [B] int32, bonus [B] int32) as CUDA
+        tensors, plus (node_p [B,N+1] f32, stats [B,4] int32) when ``debug``.
+        Asynchronous on ``stream`` (default: torch's current stream)."""
+        import torch
+        B, N = self._check(parents, tokens, logits, drafts, uniforms)
+        if out is None:
+            path = torch.empty(B, N, dtype=torch.int32, device=self.device)
+            tau = torch.empty(B, dtype=torch.int32, device=self.device)
+            bonus = torch.empty(B, dtype=torch.int32, device=self.device)
+        else:
+            path, tau, bonus = out
+        sp = _stream_ptr(stream)
+        if debug:
+            node_p = torch.empty(B, N + 1, dtype=torch.float32, device=self.device)
+            stats = torch.empty(B, 4, dtype=torch.int32, device=self.device)
+            rc = self.lib.tv_verify_batch_debug(
+                self.handle, B, N, _ptr(parents), _ptr(tokens), _ptr(logits), _ptr(drafts),
+                float(temperature), _ptr(uniforms), _ptr(path), _ptr(tau), _ptr(bonus),
+                _ptr(node_p), _ptr(stats), sp)
+            if rc != 0:
+                raise LibraryError("tv_verify_batch_debug", rc, self.lib)
+            return path, tau, bonus, node_p, stats
+        rc = self.lib.tv_verify_batch(
+            self.handle, B, N, _ptr(parents), _ptr(tokens), _ptr(logits), _ptr(drafts),
+            float(temperature), _ptr(uniforms), _ptr(path), _ptr(tau), _ptr(bonus), sp)
+        if rc != 0:
+            raise LibraryError("tv_verify_batch", rc, self.lib)
+        return path, tau, bonus
+
+    def verify_host(self, parents, tokens, logits, drafts, temperature, uniforms,
+                    out, stream=None):
+        """Same verification from host (CPU, ideally pinned) tensors; copies in,
+        verifies, copies the outputs into ``out`` = (path, tau, bonus) host
+        tensors and synchronises."""
+        B, R = parents.shape
+        N = R - 1
+        path, tau, bonus = out
+        rc = self.lib.tv_verify_batch_host(
+            self.handle, B, N, _ptr(parents), _ptr(tokens), _ptr(logits), _ptr(drafts),
+            float(temperature), _ptr(uniforms), _ptr(path), _ptr(tau), _ptr(bonus),
+            _stream_ptr(stream))
+        if rc != 0:
+            raise LibraryError("tv_verify_batch_host", rc, self.lib)
+        return path, tau, bonus
+
+    def set_phase_timing(self, enable=True):
+        rc = self.lib.tv_set_phase_timing(self.handle, 1 if enable else 0)
+        if rc != 0:
+            raise LibraryError("tv_set_phase_timing", rc, self.lib)
+
+    def last_phase_ms(self):
+        """Device milliseconds of (prep, row normalisers, traversal) of the
+        last call made with phase timing on (waits for it)."""
+        ms = (ctypes.c_float * 3)()
+        rc = self.lib.tv_last_phase_ms(self.handle, ms)
+        if rc != 0:
+            raise LibraryError("tv_last_phase_ms", rc, self.lib)
+        return [float(x) for x in ms]
+
+    def status(self):
+        """Synchronise and return (and clear) the TV_STATUS_* bits raised."""
+        v = ctypes.c_uint32(0)
+        rc = self.lib.tv_get_status(self.handle, ctypes.byref(v))
+        if rc != 0:
+            raise LibraryError("tv_get_status", rc, self.lib)
+        return v.value

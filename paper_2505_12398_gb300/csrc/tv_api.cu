@@ -1,0 +1,340 @@
+// tv_api.cu -- host side of the C ABI declared in include/tv.h.
+//
+// Argument checks happen here, before anything is queued; the kernels and
+// their launch sequence live in tv_kernels.cu.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+#include <cstdlib>
+#include <new>
+
+#include "../../include/tv.h"
+#include "tv_launch.h"
+
+struct tv_handle {
+  int device = 0;
+  int vocab = 0;
+  int max_nodes = 0;
+  int max_batch = 0;
+  tv_dtype dtype = TV_BF16;
+  unsigned flags = 0;
+  int sm_count = 0;
+  // device workspace
+  int32_t* row_list = nullptr;   // [max_batch * (max_nodes + 1)]
+  int32_t* n_rows = nullptr;     // [1]
+  float2* stats = nullptr;       // [max_batch * (max_nodes + 1)]
+  uint32_t* status = nullptr;    // [1]
+  // staging for tv_verify_batch_host (allocated on first use)
+  char* stage = nullptr;
+  size_t stage_bytes = 0;
+  // optional per-kernel timing events
+  bool timing = false;
+  bool timed_call = false;
+  cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
+};
+
+namespace {
+
+constexpr int kMaxRows = 1024;   // N + 1
+constexpr int kMaxVocab = 1 << 28;
+
+class DeviceGuard {
+ public:
+  explicit DeviceGuard(int dev) {
+    ok_ = cudaGetDevice(&prev_) == cudaSuccess;
+    if (ok_ && prev_ != dev) ok_ = cudaSetDevice(dev) == cudaSuccess;
+    switched_ = ok_ && prev_ != dev;
+  }
+  ~DeviceGuard() {
+    if (switched_) cudaSetDevice(prev_);
+  }
+  bool ok() const { return ok_; }
+
+ private:
+  int prev_ = 0;
+  bool ok_ = false;
+  bool switched_ = false;
+};
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+size_t logit_bytes(const tv_handle* h) { return h->dtype == TV_BF16 ? 2 : 4; }
+
+int check_call(const tv_handle* h, int B, int N, const void* parents, const void* tokens,
+               const void* logits, const void* drafts, float temperature,
+               const void* uniforms, const void* out_path, const void* out_len,
+               const void* out_bonus, bool device_arrays = true) {
+  if (!h) return TV_ERR_INVALID_ARG;
+  if (B < 0 || N < 0) return TV_ERR_INVALID_ARG;
+  if (B > h->max_batch || N > h->max_nodes) return TV_ERR_CAPACITY;
+  if (!(std::isfinite(temperature) && temperature > 0.f)) return TV_ERR_TEMPERATURE;
+  if (B == 0) return TV_OK;
+  if (!parents || !tokens || !logits || !drafts || !uniforms || !out_len || !out_bonus)
+    return TV_ERR_INVALID_ARG;
+  if (N > 0 && !out_path) return TV_ERR_INVALID_ARG;
+  if (device_arrays && (!aligned16(logits) || !aligned16(drafts))) return TV_ERR_INVALID_ARG;
+  return TV_OK;
+}
+
+int verify_impl(tv_handle* h, int B, int N, const int32_t* parents, const int32_t* tokens,
+                const void* logits, const float* drafts, float temperature,
+                const float* uniforms, int32_t* out_path, int32_t* out_len, int32_t* out_bonus,
+                float* out_node_p, int32_t* out_stats, void* stream) {
+  int rc = check_call(h, B, N, parents, tokens, logits, drafts, temperature, uniforms,
+                      out_path, out_len, out_bonus);
+  if (rc != TV_OK || B == 0) return rc;
+  DeviceGuard guard(h->device);
+  if (!guard.ok()) return TV_ERR_CUDA;
+  TravArgs a;
+  a.parents = parents;
+  a.tokens = tokens;
+  a.logits = logits;
+  a.draft_probs = drafts;
+  a.uniforms = uniforms;
+  a.stats = h->stats;
+  a.B = B;
+  a.N = N;
+  a.V = h->vocab;
+  a.cT = static_cast<float>(1.4426950408889634 / static_cast<double>(temperature));
+  a.out_path = out_path;
+  a.out_accept_len = out_len;
+  a.out_bonus = out_bonus;
+  a.out_node_p = out_node_p;
+  a.out_stats = out_stats;
+  a.status = h->status;
+  const int rows = B * (N + 1);
+  int grid = h->sm_count * 4;
+  if (grid > rows) grid = rows;
+  if (grid < 1) grid = 1;
+  rc = tv_launch_all(a, h->dtype == TV_BF16 ? 1 : 0, h->row_list, h->n_rows, grid,
+                     static_cast<cudaStream_t>(stream), h->timing ? h->ev : nullptr);
+  if (rc == TV_OK && h->timing) h->timed_call = true;
+  return rc;
+}
+
+}  // namespace
+
+extern "C" {
+
+int tv_create(tv_handle** out, int device, int vocab, int max_nodes, int max_batch,
+              tv_dtype logit_dtype, unsigned flags) {
+  if (!out) return TV_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (vocab < 1 || vocab > kMaxVocab) return TV_ERR_VOCAB;
+  if (max_nodes < 0 || max_nodes + 1 > kMaxRows || max_batch < 1) return TV_ERR_INVALID_ARG;
+  if (logit_dtype != TV_BF16 && logit_dtype != TV_FP32) return TV_ERR_INVALID_ARG;
+  if (flags != TV_FLAG_NONE) return TV_ERR_INVALID_ARG;
+  int ndev = 0;
+  if (cudaGetDeviceCount(&ndev) != cudaSuccess || device < 0 || device >= ndev) {
+    cudaGetLastError();
+    return TV_ERR_CUDA;
+  }
+  cudaDeviceProp prop;
+  if (cudaGetDeviceProperties(&prop, device) != cudaSuccess) return TV_ERR_CUDA;
+  if (prop.major < 10) return TV_ERR_DEVICE;
+  const size_t smem = tv_traverse_smem_bytes(max_nodes + 1, vocab);
+  if (smem > static_cast<size_t>(prop.sharedMemPerBlockOptin)) return TV_ERR_VOCAB;
+
+  tv_handle* h = new (std::nothrow) tv_handle;
+  if (!h) return TV_ERR_CUDA;
+  h->device = device;
+  h->vocab = vocab;
+  h->max_nodes = max_nodes;
+  h->max_batch = max_batch;
+  h->dtype = logit_dtype;
+  h->flags = flags;
+  h->sm_count = prop.multiProcessorCount;
+  DeviceGuard guard(device);
+  if (!guard.ok()) {
+    delete h;
+    return TV_ERR_CUDA;
+  }
+  const size_t rows = static_cast<size_t>(max_batch) * (max_nodes + 1);
+  bool ok = cudaMalloc(&h->row_list, rows * sizeof(int32_t)) == cudaSuccess &&
+            cudaMalloc(&h->n_rows, sizeof(int32_t)) == cudaSuccess &&
+            cudaMalloc(&h->stats, rows * sizeof(float2)) == cudaSuccess &&
+            cudaMalloc(&h->status, sizeof(uint32_t)) == cudaSuccess &&
+            cudaMemset(h->status, 0, sizeof(uint32_t)) == cudaSuccess;
+  if (!ok) {
+    cudaGetLastError();
+    tv_destroy(h);
+    return TV_ERR_CUDA;
+  }
+  *out = h;
+  return TV_OK;
+}
+
+int tv_verify_batch(tv_handle* h, int B, int N, const int32_t* parents,
+                    const int32_t* draft_tokens, const void* target_logits,
+                    const float* draft_probs, float temperature, const float* uniforms,
+                    int32_t* out_accepted_path, int32_t* out_accept_len,
+                    int32_t* out_bonus_token, void* cuda_stream) {
+  return verify_impl(h, B, N, parents, draft_tokens, target_logits, draft_probs, temperature,
+                     uniforms, out_accepted_path, out_accept_len, out_bonus_token, nullptr,
+                     nullptr, cuda_stream);
+}
+
+int tv_verify_batch_debug(tv_handle* h, int B, int N, const int32_t* parents,
+                          const int32_t* draft_tokens, const void* target_logits,
+                          const float* draft_probs, float temperature,
+                          const float* uniforms, int32_t* out_accepted_path,
+                          int32_t* out_accept_len, int32_t* out_bonus_token,
+                          float* out_node_p, int32_t* out_stats, void* cuda_stream) {
+  return verify_impl(h, B, N, parents, draft_tokens, target_logits, draft_probs, temperature,
+                     uniforms, out_accepted_path, out_accept_len, out_bonus_token, out_node_p,
+                     out_stats, cuda_stream);
+}
+
+int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
+                         const int32_t* draft_tokens, const void* target_logits,
+                         const float* draft_probs, float temperature,
+                         const float* uniforms, int32_t* out_accepted_path,
+                         int32_t* out_accept_len, int32_t* out_bonus_token,
+                         void* cuda_stream) {
+  int rc = check_call(h, B, N, parents, draft_tokens, target_logits, draft_probs, temperature,
+                      uniforms, out_accepted_path, out_accept_len, out_bonus_token, false);
+  if (rc != TV_OK || B == 0) return rc;
+  DeviceGuard guard(h->device);
+  if (!guard.ok()) return TV_ERR_CUDA;
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  const size_t R = static_cast<size_t>(N) + 1;
+  const size_t V = static_cast<size_t>(h->vocab);
+  const size_t n_tree = static_cast<size_t>(B) * R * sizeof(int32_t);
+  const size_t n_logit = static_cast<size_t>(B) * R * V * logit_bytes(h);
+  const size_t n_draft = static_cast<size_t>(B) * R * V * sizeof(float);
+  const size_t n_unif = static_cast<size_t>(B) * (R + 1) * sizeof(float);
+  const size_t n_path = static_cast<size_t>(B) * N * sizeof(int32_t);
+  const size_t n_out = static_cast<size_t>(B) * sizeof(int32_t);
+  auto up = [](size_t x) { return (x + 255) & ~static_cast<size_t>(255); };
+  const size_t need = up(n_logit) + up(n_draft) + 2 * up(n_tree) + up(n_unif) + up(n_path) +
+                      2 * up(n_out);
+  if (need > h->stage_bytes) {
+    // sized for the handle's limits so that later calls never reallocate
+    const size_t Rm = static_cast<size_t>(h->max_nodes) + 1;
+    const size_t Bm = static_cast<size_t>(h->max_batch);
+    const size_t cap = up(Bm * Rm * V * logit_bytes(h)) + up(Bm * Rm * V * 4) +
+                       2 * up(Bm * Rm * 4) + up(Bm * (Rm + 1) * 4) + up(Bm * (Rm - 1) * 4) +
+                       2 * up(Bm * 4);
+    if (h->stage) cudaFree(h->stage);
+    h->stage = nullptr;
+    h->stage_bytes = 0;
+    if (cudaMalloc(&h->stage, cap) != cudaSuccess) {
+      cudaGetLastError();
+      return TV_ERR_CUDA;
+    }
+    h->stage_bytes = cap;
+  }
+  char* p = h->stage;
+  void* d_logit = p; p += up(n_logit);
+  float* d_draft = reinterpret_cast<float*>(p); p += up(n_draft);
+  int32_t* d_par = reinterpret_cast<int32_t*>(p); p += up(n_tree);
+  int32_t* d_tok = reinterpret_cast<int32_t*>(p); p += up(n_tree);
+  float* d_unif = reinterpret_cast<float*>(p); p += up(n_unif);
+  int32_t* d_path = reinterpret_cast<int32_t*>(p); p += up(n_path);
+  int32_t* d_len = reinterpret_cast<int32_t*>(p); p += up(n_out);
+  int32_t* d_bonus = reinterpret_cast<int32_t*>(p);
+  bool ok = cudaMemcpyAsync(d_par, parents, n_tree, cudaMemcpyHostToDevice, st) == cudaSuccess &&
+            cudaMemcpyAsync(d_tok, draft_tokens, n_tree, cudaMemcpyHostToDevice, st) == cudaSuccess &&
+            cudaMemcpyAsync(d_unif, uniforms, n_unif, cudaMemcpyHostToDevice, st) == cudaSuccess &&
+            cudaMemcpyAsync(d_logit, target_logits, n_logit, cudaMemcpyHostToDevice, st) == cudaSuccess &&
+            cudaMemcpyAsync(d_draft, draft_probs, n_draft, cudaMemcpyHostToDevice, st) == cudaSuccess;
+  if (!ok) {
+    cudaGetLastError();
+    return TV_ERR_CUDA;
+  }
+  rc = verify_impl(h, B, N, d_par, d_tok, d_logit, d_draft, temperature, d_unif, d_path, d_len,
+                   d_bonus, nullptr, nullptr, cuda_stream);
+  if (rc != TV_OK) return rc;
+  ok = (N == 0 || cudaMemcpyAsync(out_accepted_path, d_path, n_path, cudaMemcpyDeviceToHost, st) ==
+                      cudaSuccess) &&
+       cudaMemcpyAsync(out_accept_len, d_len, n_out, cudaMemcpyDeviceToHost, st) == cudaSuccess &&
+       cudaMemcpyAsync(out_bonus_token, d_bonus, n_out, cudaMemcpyDeviceToHost, st) == cudaSuccess &&
+       cudaStreamSynchronize(st) == cudaSuccess;
+  if (!ok) {
+    cudaGetLastError();
+    return TV_ERR_CUDA;
+  }
+  return TV_OK;
+}
+
+int tv_get_status(tv_handle* h, uint32_t* status) {
+  if (!h || !status) return TV_ERR_INVALID_ARG;
+  DeviceGuard guard(h->device);
+  if (!guard.ok()) return TV_ERR_CUDA;
+  uint32_t v = 0;
+  if (cudaDeviceSynchronize() != cudaSuccess ||
+      cudaMemcpy(&v, h->status, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess ||
+      cudaMemset(h->status, 0, sizeof(uint32_t)) != cudaSuccess) {
+    cudaGetLastError();
+    return TV_ERR_CUDA;
+  }
+  *status = v;
+  return TV_OK;
+}
+
+int tv_set_phase_timing(tv_handle* h, int enable) {
+  if (!h) return TV_ERR_INVALID_ARG;
+  DeviceGuard guard(h->device);
+  if (!guard.ok()) return TV_ERR_CUDA;
+  if (enable && !h->ev[0]) {
+    for (int k = 0; k < 4; ++k) {
+      if (cudaEventCreate(&h->ev[k]) != cudaSuccess) {
+        cudaGetLastError();
+        return TV_ERR_CUDA;
+      }
+    }
+  }
+  h->timing = enable != 0;
+  h->timed_call = false;
+  return TV_OK;
+}
+
+int tv_last_phase_ms(tv_handle* h, float* ms) {
+  if (!h || !ms || !h->timing || !h->timed_call) return TV_ERR_INVALID_ARG;
+  DeviceGuard guard(h->device);
+  if (!guard.ok()) return TV_ERR_CUDA;
+  if (cudaEventSynchronize(h->ev[3]) != cudaSuccess) return TV_ERR_CUDA;
+  for (int k = 0; k < 3; ++k) {
+    if (cudaEventElapsedTime(&ms[k], h->ev[k], h->ev[k + 1]) != cudaSuccess) {
+      cudaGetLastError();
+      return TV_ERR_CUDA;
+    }
+  }
+  return TV_OK;
+}
+
+int tv_destroy(tv_handle* h) {
+  if (!h) return TV_ERR_INVALID_ARG;
+  {
+    DeviceGuard guard(h->device);
+    if (guard.ok()) cudaDeviceSynchronize();
+    for (int k = 0; k < 4; ++k)
+      if (h->ev[k]) cudaEventDestroy(h->ev[k]);
+    cudaFree(h->row_list);
+    cudaFree(h->n_rows);
+    cudaFree(h->stats);
+    cudaFree(h->status);
+    if (h->stage) cudaFree(h->stage);
+    cudaGetLastError();
+  }
+  delete h;
+  return TV_OK;
+}
+
+const char* tv_strerror(int code) {
+  switch (code) {
+    case TV_OK: return "success";
+    case TV_ERR_INVALID_ARG: return "invalid argument (null pointer, bad size or flag, misaligned array)";
+    case TV_ERR_TEMPERATURE: return "temperature must be finite and > 0";
+    case TV_ERR_VOCAB: return "vocabulary size out of range for this device";
+    case TV_ERR_CAPACITY: return "batch or node count above the handle's limits";
+    case TV_ERR_CUDA: return "CUDA runtime error";
+    case TV_ERR_DEVICE: return "unsupported device (needs compute capability 10.x or newer)";
+    default: return "unknown error code";
+  }
+}
+
+int tv_version(void) { return 100; }
+
+}  // extern "C"

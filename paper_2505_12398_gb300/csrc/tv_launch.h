@@ -1,0 +1,32 @@
+// tv_launch.h -- internal interface between the host API and the kernels.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+struct TravArgs {
+  const int32_t* parents;      // [B][N+1]
+  const int32_t* tokens;       // [B][N+1]
+  const void* logits;          // [B][N+1][V] bf16 or fp32
+  const float* draft_probs;    // [B][N+1][V]
+  const float* uniforms;       // [B][N+2]
+  float2* stats;               // [B][N+1] row (max, sum of exp2) of internal rows
+  int B, N, V;
+  float cT;                    // log2(e) / temperature
+  int32_t* out_path;           // [B][N]
+  int32_t* out_accept_len;     // [B]
+  int32_t* out_bonus;          // [B]
+  float* out_node_p;           // [B][N+1] or nullptr
+  int32_t* out_stats;          // [B][4] or nullptr
+  uint32_t* status;            // status word (OR of TV_STATUS_* bits)
+};
+
+// Dynamic shared memory the traversal kernel needs for R = N+1 rows.
+size_t tv_traverse_smem_bytes(int R, int V);
+
+// Queues the three kernels on `stream`; 0 on success, TV_ERR_CUDA otherwise.
+// With `events` non-null, events[0..3] are recorded before the first kernel,
+// between the kernels and after the last one.
+int tv_launch_all(const TravArgs& a, int logit_is_bf16, int* row_list, int* n_rows,
+                  int stats_grid, cudaStream_t stream, cudaEvent_t* events);

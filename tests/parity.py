@@ -1,0 +1,108 @@
+"""Element-by-element comparison of the CUDA path with the CPU oracle.
+
+Decisions (accept / reject of each tested node, the bonus token) are floating
+point deciding integers: the oracle takes them in float64, the kernels in
+float32.  A tree is compared bit-exactly when every decision margin of the
+oracle (|u - p| for each test, the distance of u W to the nearest CDF step
+for the bonus, relative to W) is at least ``TIE`` = 1e-5; trees with a
+near-tie are counted, compared up to the tie, and the GPU's choice at the tie
+is checked to be a valid one within the float32 error bound.
+
+Acceptance rates p of the tested nodes must agree within
+``P_RTOL`` * p + ``P_ATOL``.
+"""
+
+import numpy as np
+
+TIE = 1e-5
+P_RTOL = 1e-5
+P_ATOL = 1e-7
+
+
+def to_numpy_inputs(inp, trees=None):
+    """Host copies (float32 logits) of a workloads.synth.Inputs batch."""
+    sel = slice(None) if trees is None else list(trees)
+    par = inp.parents[sel].cpu().numpy()
+    tok = inp.tokens[sel].cpu().numpy()
+    lg = inp.logits[sel].float().cpu().numpy()
+    dp = inp.draft_probs[sel].cpu().numpy()
+    un = inp.uniforms[sel].cpu().numpy()
+    return par, tok, lg, dp, un
+
+
+def compare_tree(r, g_path, g_tau, g_bonus, g_p=None, g_stats=None):
+    """Compare one tree; returns a dict of findings (raises nothing)."""
+    out = {"exact": False, "tie": False, "ok": True, "why": [], "max_p_rel": 0.0}
+    if "invalid" in r:
+        ok = g_tau == -1 and g_bonus == -1 and (np.asarray(g_path) == -1).all()
+        out.update(exact=ok, ok=ok)
+        if not ok:
+            out["why"].append("invalid tree not marked")
+        return out
+    tests = r["tests"]
+    tie_at = None
+    for k, (node, u, p) in enumerate(tests):
+        if abs(u - p) < TIE:
+            tie_at = k
+            break
+    n_cmp = len(tests) if tie_at is None else tie_at + 1
+    if g_p is not None:
+        for node, u, p in tests[:n_cmp]:
+            gp = float(g_p[node])
+            err = abs(gp - p)
+            if p > 0:
+                out["max_p_rel"] = max(out["max_p_rel"], err / p)
+            if not err <= P_RTOL * p + P_ATOL:
+                out["ok"] = False
+                out["why"].append(f"p of node {node}: gpu {gp!r} oracle {p!r}")
+        for c in r["pruned"]:
+            if tie_at is None and float(g_p[c]) != 0.0:
+                out["ok"] = False
+                out["why"].append(f"pruned node {c} has gpu p {g_p[c]}")
+    if tie_at is not None:
+        out["tie"] = True
+        return out
+    path = list(np.asarray(g_path)[: max(g_tau, 0)])
+    if g_tau != r["tau"] or path != r["path"]:
+        out["ok"] = False
+        out["why"].append(f"path gpu {path} (tau {g_tau}) oracle {r['path']} (tau {r['tau']})")
+        return out
+    if g_stats is not None:
+        want = [len(tests), r["n_passes"], len(r["rejected_at"]), int(r["leaf_row_read"])]
+        if list(np.asarray(g_stats)) != want:
+            out["ok"] = False
+            out["why"].append(f"stats gpu {list(g_stats)} oracle {want}")
+    if r["bonus_margin"] < TIE:
+        out["tie"] = True
+        cdf = r.get("bonus_cdf")
+        if cdf is not None:
+            W = cdf[-1]
+            t = r["bonus_u"] * W
+            y = int(g_bonus)
+            lo = cdf[y - 1] if y > 0 else 0.0
+            if not (0 <= y < len(cdf) and lo - TIE * W <= t < cdf[y] + TIE * W):
+                out["ok"] = False
+                out["why"].append(f"bonus {y} outside the near-tie band")
+        return out
+    if g_bonus != r["bonus"]:
+        out["ok"] = False
+        out["why"].append(f"bonus gpu {g_bonus} oracle {r['bonus']}")
+        return out
+    out["exact"] = True
+    return out
+
+
+def compare_batch(details, g_path, g_tau, g_bonus, g_p=None, g_stats=None):
+    """details: {tree index: oracle result}.  Returns summary dict."""
+    summ = {"trees": 0, "exact": 0, "ties": 0, "bad": [], "max_p_rel": 0.0}
+    for b, r in details.items():
+        c = compare_tree(r, g_path[b], int(g_tau[b]), int(g_bonus[b]),
+                         None if g_p is None else g_p[b],
+                         None if g_stats is None else g_stats[b])
+        summ["trees"] += 1
+        summ["exact"] += int(c["exact"])
+        summ["ties"] += int(c["tie"])
+        summ["max_p_rel"] = max(summ["max_p_rel"], c["max_p_rel"])
+        if not c["ok"]:
+            summ["bad"].append((b, c["why"]))
+    return summ

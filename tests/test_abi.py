@@ -1,0 +1,56 @@
+"""CPU checks of the boundary: the shared library builds, loads, and exports
+every entry point include/tv.h declares (no GPU needed, no compute calls)."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "tv.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(tv_[a-z_]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2505_12398_gb300.build import build
+    path = build()
+    return ctypes.CDLL(path)
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for need in ("tv_create", "tv_verify_batch", "tv_destroy"):
+        assert need in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_error_strings_and_version(lib):
+    lib.tv_strerror.restype = ctypes.c_char_p
+    for code in (0, -1, -2, -3, -4, -5, -6):
+        assert lib.tv_strerror(code) and lib.tv_strerror(code) != b"unknown error code"
+    assert lib.tv_strerror(-99) == b"unknown error code"
+    assert lib.tv_version() >= 100
+
+
+def test_binding_signatures_cover_the_header():
+    from paper_2505_12398_gb300._binding import _SIGS
+    assert set(_SIGS) == set(declared_functions())
+
+
+def test_product_path_does_not_import_the_oracle():
+    pkg = os.path.join(ROOT, "paper_2505_12398_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h")):
+                text = open(os.path.join(dirpath, f)).read()
+                assert "import oracle" not in text and "from oracle" not in text, f

@@ -1,0 +1,174 @@
+"""GPU parity: the CUDA path against the CPU oracle on the same seeded inputs
+and the same pre-drawn uniforms, element by element (see tests/parity.py for
+the comparison rule and tolerances).  All calls go through the C ABI."""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle.verify import verify_batch
+from tests.parity import compare_batch, to_numpy_inputs
+from workloads.synth import get_workload, make_inputs
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def tv():
+    import paper_2505_12398_gb300 as tv
+    from paper_2505_12398_gb300.build import build
+    build()
+    return tv
+
+
+def run_gpu(tv, inp, debug=True):
+    B, R = inp.parents.shape
+    V = inp.logits.shape[-1]
+    dt = "bf16" if inp.logits.dtype == torch.bfloat16 else "fp32"
+    v = tv.Verifier(V, R - 1, B, dt)
+    out = v.verify(inp.parents, inp.tokens, inp.logits, inp.draft_probs, inp.temperature,
+                   inp.uniforms, debug=debug)
+    torch.cuda.synchronize()
+    status = v.status()
+    v.close()
+    return [o.cpu().numpy() for o in out], status
+
+
+def check(tv, inp, trees=None, max_tie_frac=0.25):
+    (path, tau, bonus, node_p, stats), status = run_gpu(tv, inp)
+    if trees is None:
+        trees = list(range(inp.parents.shape[0]))
+    par, tok, lg, dp, un = to_numpy_inputs(inp, trees)
+    _, _, _, det = verify_batch(par, tok, lg, dp, inp.temperature, un, keep_cdf=True)
+    det = {trees[k]: r for k, r in det.items()}
+    summ = compare_batch(det, path, tau, bonus, node_p, stats)
+    print(f"\n{inp.meta}: trees {summ['trees']} exact {summ['exact']} "
+          f"ties {summ['ties']} max p rel err {summ['max_p_rel']:.2e}")
+    assert not summ["bad"], summ["bad"][:5]
+    assert summ["ties"] <= max_tie_frac * summ["trees"] + 1
+    return summ, status
+
+
+def test_tiny_many_seeds(tv):
+    """The 7-node, V=64, fp32 tree, 512 draws of logits / tree / uniforms."""
+    w = get_workload("tiny", batch=512)
+    inp = make_inputs(w, seed=0, device="cuda")
+    summ, status = check(tv, inp)
+    assert summ["exact"] >= 0.9 * summ["trees"]
+    assert status & ~16 == 0
+
+
+@pytest.mark.parametrize("name", ["chain8", "binary4"])
+@pytest.mark.parametrize("sigma", [0.5, 1.0, 2.0])
+def test_chain_and_binary(tv, name, sigma):
+    w = get_workload(name, sigma=sigma)
+    inp = make_inputs(w, seed=1, device="cuda")
+    check(tv, inp)
+
+
+def test_eagle_v32k_all_trees(tv):
+    w = get_workload("eagle_v32k")
+    inp = make_inputs(w, seed=2, device="cuda")
+    check(tv, inp)
+
+
+def test_eagle_v128k_sampled(tv):
+    """Full batch of 128 trees at V=128256 (the benchmark workload); the
+    oracle checks a sample of 12 trees."""
+    w = get_workload("eagle_v128k")
+    inp = make_inputs(w, seed=3, device="cuda")
+    trees = list(range(0, 128, 11))
+    check(tv, inp, trees=trees)
+
+
+@pytest.mark.parametrize("V", [1000, 1003, 257, 8])
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_ragged_vocab(tv, V, dtype):
+    """Vocabularies that are not a multiple of the 8-element chunk or of the
+    256-element bonus tile exercise the scalar-load path and the tails."""
+    from workloads.synth import Workload
+    w = Workload("ragged", 48, V, levels=(2, 3, 2), branching=(2, 2, 1),
+                 logit_dtype=dtype, sigma=1.0)
+    inp = make_inputs(w, seed=V, device="cuda")
+    check(tv, inp)
+
+
+def test_root_only_trees(tv):
+    from workloads.synth import Workload
+    w = Workload("root_only", 32, 5000, parents=(-1,), logit_dtype=torch.bfloat16)
+    inp = make_inputs(w, seed=5, device="cuda")
+    (path, tau, bonus, node_p, stats), status = run_gpu(tv, inp)
+    par, tok, lg, dp, un = to_numpy_inputs(inp)
+    _, otau, obonus, det = verify_batch(par, tok, lg, dp, inp.temperature, un)
+    assert (tau == 0).all()
+    near = np.array([det[b]["bonus_margin"] < 1e-5 for b in range(32)])
+    assert (bonus[~near] == obonus[~near]).all()
+
+
+@pytest.mark.parametrize("T", [0.2, 2.0])
+def test_temperatures(tv, T):
+    from workloads.synth import Workload
+    w = Workload("temp", 24, 4096, levels=(3, 6, 6, 4), branching=(3, 2, 1, 1),
+                 logit_dtype=torch.bfloat16, temperature=T)
+    inp = make_inputs(w, seed=int(T * 10), device="cuda")
+    check(tv, inp)
+
+
+def test_invalid_trees_flagged(tv):
+    from workloads.synth import Workload
+    w = Workload("inv", 6, 512, levels=(2, 2), branching=(2, 1), logit_dtype=torch.float32)
+    inp = make_inputs(w, seed=9, device="cuda")
+    inp.parents[1, 2] = 3            # parent after child
+    inp.tokens[2, 2] = inp.tokens[2, 1]   # duplicate siblings
+    inp.tokens[3, 4] = 512           # outside the vocabulary
+    inp.parents[4, 0] = 0            # root with a parent
+    par = inp.parents[5].tolist()
+    inp.draft_probs[5, par[1], inp.tokens[5, 1]] = 0.0   # zero draft probability
+    (path, tau, bonus, node_p, stats), status = run_gpu(tv, inp)
+    assert tau[0] >= 0
+    assert (tau[1:] == -1).all() and (bonus[1:] == -1).all() and (path[1:] == -1).all()
+    assert status & 1 and status & 2 and status & 4 and status & 8
+    p2, t2, l2, d2, u2 = to_numpy_inputs(inp)
+    _, otau, _, _ = verify_batch(p2, t2, l2, d2, inp.temperature, u2)
+    assert (otau[1:] == -1).all()
+
+
+def test_host_entry_point_matches_device(tv):
+    w = get_workload("binary4", batch=8)
+    inp = make_inputs(w, seed=4, device="cuda")
+    (path, tau, bonus, _, _), _ = run_gpu(tv, inp)
+    B, R = inp.parents.shape
+    v = tv.Verifier(w.vocab, R - 1, B, "fp32")
+    hp = [inp.parents.cpu(), inp.tokens.cpu(), inp.logits.cpu(), inp.draft_probs.cpu(),
+          inp.uniforms.cpu()]
+    out = (torch.empty(B, R - 1, dtype=torch.int32), torch.empty(B, dtype=torch.int32),
+           torch.empty(B, dtype=torch.int32))
+    v.verify_host(hp[0], hp[1], hp[2], hp[3], inp.temperature, hp[4], out)
+    v.close()
+    assert (out[0].numpy() == path).all() and (out[1].numpy() == tau).all()
+    assert (out[2].numpy() == bonus).all()
+
+
+def test_host_argument_errors(tv):
+    w = get_workload("tiny", batch=2)
+    inp = make_inputs(w, seed=0, device="cuda")
+    v = tv.Verifier(64, 7, 2, "fp32")
+    with pytest.raises(tv.LibraryError) as e:
+        v.verify(inp.parents, inp.tokens, inp.logits, inp.draft_probs, 0.0, inp.uniforms)
+    assert e.value.code == -2
+    with pytest.raises(tv.LibraryError) as e:
+        v.verify(inp.parents, inp.tokens, inp.logits, inp.draft_probs, float("nan"),
+                 inp.uniforms)
+    assert e.value.code == -2
+    v.close()
+    small = tv.Verifier(64, 3, 2, "fp32")
+    rc = small.lib.tv_verify_batch(small.handle, 2, 7, None, None, None, None, 1.0, None,
+                                   None, None, None, None)
+    assert rc == -4
+    rc = small.lib.tv_verify_batch(small.handle, 1, 3, None, None, None, None, 1.0, None,
+                                   None, None, None, None)
+    assert rc == -1
+    rc = small.lib.tv_verify_batch(small.handle, 0, 3, None, None, None, None, 1.0, None,
+                                   None, None, None, None)
+    assert rc == 0
+    small.close()
