@@ -121,6 +121,24 @@ def validate_tree(parents, tokens, vocab, allow_duplicate_siblings=False):
             seen[key] = i
 
 
+def _condition(p, mb, ms, S):
+    """Instrumentation only: relative sensitivity of S to relative
+    perturbations of M_b, sum over the positive part of p M_b(x), divided by
+    S (inf when S = 0).  A float computation of S whose M_b values carry a
+    relative error e has a relative error of about e times this number."""
+    pos = (p * mb - ms) > 0
+    if not S > 0:
+        return float("inf")
+    return float((p * mb)[pos].sum() / S)
+
+
+def _cancellation(u, v):
+    """Instrumentation only: condition number (|u| + |v|) / |u - v| of u - v."""
+    diff = abs(float(u) - float(v))
+    tot = abs(float(u)) + abs(float(v))
+    return float("inf") if diff == 0 else tot / diff
+
+
 class TraversalState:
     """Mutable state of Algorithm 3 on one decoding tree.
 
@@ -161,6 +179,7 @@ class TraversalState:
         # instrumentation: S-computations per node, degenerate S == 0 events,
         # nodes removed with rate 0, and the bonus row fetched for a leaf
         self.passes = [0] * n
+        self.kappa = []         # condition number of each S (instrumentation)
         self.degenerate = 0
         self.pruned = []
         self.leaf_rows_read = set()
@@ -232,9 +251,16 @@ class TraversalState:
         mb, ms = self.mb[i], self.ms[i]
         S = residual_mass(p, mb, ms)
         self.passes[i] += 1
+        self.kappa.append(_condition(p, mb, ms, S))
         if S > 0:
             new_mb = residual_target(p, mb, ms, S)
             new_p = updated_rate(p, S)
+            # instrumentation: cancellation in the residual of every remaining
+            # child's token, on top of that of S
+            for d in self.children[i]:
+                if self.alive[d]:
+                    x = self.tokens[d]
+                    self.kappa.append(self.kappa[-1] + _cancellation(p * mb[x], ms[x]))
         else:
             self.degenerate += 1
             new_mb = mb

@@ -71,6 +71,7 @@ def verify_tree(parents, tokens, logits, draft_probs, temperature, uniforms, kee
                         vocab=V)
     node_p = np.full(n, np.nan)
     tests = []
+    kappa_at_test = []
     while True:
         leaf = st.first_leaf()
         if leaf == 0:
@@ -79,6 +80,7 @@ def verify_tree(parents, tokens, logits, draft_probs, temperature, uniforms, kee
         p = float(st.p[leaf])
         node_p[leaf] = p
         tests.append((leaf, float(u[leaf]), p))
+        kappa_at_test.append(max(st.kappa, default=1.0))
         if u[leaf] < p:
             accepted = leaf
             break
@@ -97,6 +99,7 @@ def verify_tree(parents, tokens, logits, draft_probs, temperature, uniforms, kee
         "accepted": accepted,
         "node_p": node_p,
         "tests": tests,
+        "kappa_at_test": kappa_at_test,
         "test_margin": min((abs(uu - pp) for _, uu, pp in tests), default=np.inf),
         "bonus_margin": y_margin,
         "bonus_total": W,

@@ -96,7 +96,10 @@ int verify_impl(tv_handle* h, int B, int N, const int32_t* parents, const int32_
   a.B = B;
   a.N = N;
   a.V = h->vocab;
-  a.cT = static_cast<float>(1.4426950408889634 / static_cast<double>(temperature));
+  const double c = 1.4426950408889634 / static_cast<double>(temperature);
+  a.c_hi = static_cast<float>(c);
+  a.c_lo = static_cast<float>(c - static_cast<double>(a.c_hi));
+  a.c = c;
   a.out_path = out_path;
   a.out_accept_len = out_len;
   a.out_bonus = out_bonus;

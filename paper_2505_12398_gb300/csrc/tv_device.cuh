@@ -1,11 +1,20 @@
 // tv_device.cuh -- device helpers shared by the verification kernels.
 //
-// Numerics of the GPU path (float32 throughout):
-//   M_b(x|X^i) = exp2((l_i(x) - m_i) * c) / s_i  with  c = log2(e) / T,
-// where m_i is the row's largest logit and s_i = sum_x exp2((l_i(x) - m_i) c)
-// (the softmax of l / T written in base 2, §3.1's target distributions).
-// The difference l - m is exact for bf16 inputs, so the exponent carries only
-// the rounding of one multiply; exp2 is the hardware ex2.approx instruction.
+// Numerics of the GPU path:
+//   M_b(x|X^i) = e_i(x) / s_i,  e_i(x) = 2^((l_i(x) - m_i) c),  c = log2(e) / T,
+// where m_i is the row's largest logit and s_i = sum_x e_i(x) (the softmax of
+// l / T written in base 2; the target distributions of §3.1).  Vocabulary-wide
+// work is float32; the serial control of the traversal is float64.
+//
+// e(x) is computed so that its relative error stays near one float32 ulp:
+// the exponent E = (l - m) c is formed as an unevaluated sum E_hi + E_lo
+// (c split into c_hi + c_lo, the product error recovered with an FMA), split
+// into an integer n and a fraction f in [-1/2, 1/2] with f carrying E_lo,
+// and 2^f is taken from the ex2.approx instruction on that small argument;
+// 2^n is applied by adding n to the exponent field.  Rounding the exponent of
+// a large |E| to float32 first would leave a relative error of up to
+// |E| 2^-24 ln 2 in every e(x), with a systematic sign; the rejection sum
+// S = sum_x [p M_b(x) - M_s(x)]_+ amplifies such errors when it cancels.
 #pragma once
 
 #include <cuda_runtime.h>
@@ -20,6 +29,23 @@ __device__ __forceinline__ float ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+
+// 2^E for E = d c with c = c_hi + c_lo and d = d_hi + d_lo (see above).
+__device__ __forceinline__ float exp2_split(float d, float d_lo, float c_hi, float c_lo) {
+  d = fmaxf(d, -1.0e4f);                      // -inf / NaN logits -> weight ~0
+  const float e_hi = d * c_hi;
+  float e_lo = fmaf(d, c_hi, -e_hi);          // exact error of the product
+  e_lo = fmaf(d, c_lo, e_lo);
+  e_lo = fmaf(d_lo, c_hi, e_lo);
+  const float t = e_hi + 12582912.f;          // 1.5 * 2^23: round to integer
+  const float nf = t - 12582912.f;
+  int ni = __float_as_int(t) - 0x4B400000;
+  const float f = (e_hi - nf) + e_lo;         // e_hi - nf is exact
+  const float r = ex2(f);
+  // below the normal range the weight is taken as exactly 0 (this also makes
+  // padding elements, read as -inf, contribute nothing)
+  return (ni < -125) ? 0.f : __int_as_float(__float_as_int(r) + (ni << 23));
 }
 
 // Two bf16 values packed in one 32-bit word -> float (bf16 is the upper half
@@ -39,6 +65,10 @@ __device__ __forceinline__ uint4 ld_nc16(const void* p) {
 struct Bf16Logits {
   using elem = uint16_t;
   static constexpr int kBytes = 2;
+  // 2^((v - m) c): v - m is exact for two bf16 values
+  __device__ static __forceinline__ float exp_rel(float v, float m, float c_hi, float c_lo) {
+    return exp2_split(v - m, 0.f, c_hi, c_lo);
+  }
   __device__ static __forceinline__ float at(const elem* row, int x) {
     return __uint_as_float(static_cast<uint32_t>(row[x]) << 16);
   }
@@ -55,6 +85,14 @@ struct Bf16Logits {
 struct F32Logits {
   using elem = float;
   static constexpr int kBytes = 4;
+  // 2^((v - m) c) with the rounding error of v - m carried along (two-sum)
+  __device__ static __forceinline__ float exp_rel(float v, float m, float c_hi, float c_lo) {
+    v = fmaxf(v, m - 1.0e4f);                 // -inf / NaN: finite, weight ~0
+    const float d = v - m;
+    const float bb = d - v;
+    const float d_lo = (v - (d - bb)) + (-m - bb);
+    return exp2_split(d, d_lo, c_hi, c_lo);
+  }
   __device__ static __forceinline__ float at(const elem* row, int x) { return __ldg(row + x); }
   __device__ static __forceinline__ void chunk_vec(const elem* row, int x0, float v[8]) {
     uint4 a = ld_nc16(row + x0);
@@ -119,25 +157,6 @@ __device__ __forceinline__ float warp_max(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
   return v;
-}
-
-// Merge two (max, sum-of-exp2 relative to that max) pairs.
-__device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2, float c) {
-  float M = fmaxf(m, m2);
-  if (M == TV_NEG_INF) { m = M; s = 0.f; return; }
-  float a = (m == TV_NEG_INF) ? 0.f : s * ex2((m - M) * c);
-  float b = (m2 == TV_NEG_INF) ? 0.f : s2 * ex2((m2 - M) * c);
-  m = M;
-  s = a + b;
-}
-
-__device__ __forceinline__ void warp_lse(float& m, float& s, float c) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    float m2 = __shfl_xor_sync(0xffffffffu, m, o);
-    float s2 = __shfl_xor_sync(0xffffffffu, s, o);
-    lse_merge(m, s, m2, s2, c);
-  }
 }
 
 }  // namespace tvk

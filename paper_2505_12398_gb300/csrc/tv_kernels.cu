@@ -94,15 +94,17 @@ constexpr int kStatsUnroll = 4;
 
 template <typename L, bool VEC>
 __global__ void __launch_bounds__(kStatsThreads) tv_row_stats_kernel(
-    const typename L::elem* __restrict__ logits, int V, float cT,
+    const typename L::elem* __restrict__ logits, int V, float c_hi, float c_lo,
     const int32_t* __restrict__ row_list, const int32_t* __restrict__ n_rows,
     float2* __restrict__ stats) {
-  __shared__ float s_m[kStatsThreads / 32], s_s[kStatsThreads / 32];
+  __shared__ float s_red[kStatsThreads / 32];
+  __shared__ float s_max;
   const int n = *n_rows;
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
   for (int r = blockIdx.x; r < n; r += gridDim.x) {
     const int g = row_list[r];
     const typename L::elem* row = logits + (size_t)g * V;
+    // phase 1: per-thread online max / sum relative to that max
     float m = TV_NEG_INF;
     Comp acc;
     const int step = kStatsThreads * kChunk;
@@ -116,13 +118,17 @@ __global__ void __launch_bounds__(kStatsThreads) tv_row_stats_kernel(
         float cm = fmaxf(fmaxf(fmaxf(v[u][0], v[u][1]), fmaxf(v[u][2], v[u][3])),
                          fmaxf(fmaxf(v[u][4], v[u][5]), fmaxf(v[u][6], v[u][7])));
         if (cm > m) {
-          if (m != TV_NEG_INF) { float sc = ex2((m - cm) * cT); acc.s *= sc; acc.c *= sc; }
+          if (m != TV_NEG_INF) {
+            const float sc = L::exp_rel(m, cm, c_hi, c_lo);
+            acc.s *= sc;
+            acc.c *= sc;
+          }
           m = cm;
         }
         if (m != TV_NEG_INF) {
           float t[8];
 #pragma unroll
-          for (int k = 0; k < 8; ++k) t[k] = ex2((v[u][k] - m) * cT);
+          for (int e = 0; e < 8; ++e) t[e] = L::exp_rel(v[u][e], m, c_hi, c_lo);
           acc.add(sum8(t));
         }
       }
@@ -132,27 +138,42 @@ __global__ void __launch_bounds__(kStatsThreads) tv_row_stats_kernel(
       load_logits<L, VEC>(row, x0, V, v);
       float cm = v[0];
 #pragma unroll
-      for (int k = 1; k < 8; ++k) cm = fmaxf(cm, v[k]);
+      for (int e = 1; e < 8; ++e) cm = fmaxf(cm, v[e]);
       if (cm > m) {
-        if (m != TV_NEG_INF) { float sc = ex2((m - cm) * cT); acc.s *= sc; acc.c *= sc; }
+        if (m != TV_NEG_INF) {
+          const float sc = L::exp_rel(m, cm, c_hi, c_lo);
+          acc.s *= sc;
+          acc.c *= sc;
+        }
         m = cm;
       }
       if (m != TV_NEG_INF) {
         float t[8];
 #pragma unroll
-        for (int k = 0; k < 8; ++k) t[k] = ex2((v[k] - m) * cT);
+        for (int e = 0; e < 8; ++e) t[e] = L::exp_rel(v[e], m, c_hi, c_lo);
         acc.add(sum8(t));
       }
     }
-    float s = (m == TV_NEG_INF) ? 0.f : acc.value();
-    warp_lse(m, s, cT);
-    if (lane == 0) { s_m[wid] = m; s_s[wid] = s; }
+    // phase 2: the row max, then every partial rescaled once to it and summed
+    float bm = warp_max(m);
+    if (lane == 0) s_red[wid] = bm;
     __syncthreads();
     if (wid == 0) {
-      m = (lane < kStatsThreads / 32) ? s_m[lane] : TV_NEG_INF;
-      s = (lane < kStatsThreads / 32) ? s_s[lane] : 0.f;
-      warp_lse(m, s, cT);
-      if (lane == 0) stats[g] = make_float2(m, s);
+      float x = (lane < kStatsThreads / 32) ? s_red[lane] : TV_NEG_INF;
+      x = warp_max(x);
+      if (lane == 0) s_max = x;
+    }
+    __syncthreads();
+    const float M = s_max;
+    float part = (m == TV_NEG_INF) ? 0.f : acc.value() * L::exp_rel(m, M, c_hi, c_lo);
+    part = warp_sum(part);
+    __syncthreads();
+    if (lane == 0) s_red[wid] = part;
+    __syncthreads();
+    if (wid == 0) {
+      float x = (lane < kStatsThreads / 32) ? s_red[lane] : 0.f;
+      x = warp_sum(x);
+      if (lane == 0) stats[g] = make_float2(M, x);
     }
     __syncthreads();
   }
@@ -171,29 +192,35 @@ struct Ctl {
   int cmd;
   int pass_node;      // node whose rows the next pass streams
   int nmask;          // removed tokens to skip in that pass
-  float alpha1;       // coefficient of exp2((l - m) c) in the pass
-  float beta;         // coefficient of M_s^(0) in the pass
+  float alpha1;       // coefficient of e(x) = 2^((l - m) c) in the pass
+  float beta;         // coefficient of M_s^(0)(x) in the pass
   float S;            // pass result (removed tokens excluded)
   int accepted;       // accepted node, -1 if the tree is invalid
   uint32_t bad;       // TV_STATUS_* bits found for this tree
-  float bonus_a;      // bonus weights: a * e(x) / s_i - b * q(x) (residual form)
+  float bonus_a;      // residual bonus weights: bonus_a e(x) - bonus_b q(x)
   float bonus_b;
-  int bonus_leaf;     // 1: draw from the accepted leaf's softmax
-  float W;            // total bonus weight
-  float rowmax;       // leaf bonus: the row's largest logit
-  int bonus_tile;
-  float bonus_base;   // cumulative weight before bonus_tile
+  float rowmax;
+  int bonus_y;
 };
 
+// Per-tree shared state.  The serial control keeps its scalars in float64.
 struct TravSmem {
+  double *p, *a, *b, *Z, *invZ, *m;
   int32_t *par, *tok, *first, *next, *npass, *mask_tok;
-  float *p, *gl, *gq, *a, *b, *Z, *invZ, *m, *rowm, *rows, *dbgp, *mask_val, *tsum, *tmax;
+  float *gl, *gq, *rowm, *rows, *dbgp, *mask_val, *tsum, *tmax;
   uint8_t* state;
 };
 
 __device__ __forceinline__ TravSmem carve(char* base, int R, int V) {
   TravSmem s;
-  int32_t* ip = reinterpret_cast<int32_t*>(base);
+  double* dp = reinterpret_cast<double*>(base);
+  s.p = dp; dp += R;
+  s.a = dp; dp += R;
+  s.b = dp; dp += R;
+  s.Z = dp; dp += R;
+  s.invZ = dp; dp += R;
+  s.m = dp; dp += R;
+  int32_t* ip = reinterpret_cast<int32_t*>(dp);
   s.par = ip; ip += R;
   s.tok = ip; ip += R;
   s.first = ip; ip += R;
@@ -201,19 +228,13 @@ __device__ __forceinline__ TravSmem carve(char* base, int R, int V) {
   s.npass = ip; ip += R;
   s.mask_tok = ip; ip += R;
   float* fp = reinterpret_cast<float*>(ip);
-  s.p = fp; fp += R;
   s.gl = fp; fp += R;
   s.gq = fp; fp += R;
-  s.a = fp; fp += R;
-  s.b = fp; fp += R;
-  s.Z = fp; fp += R;
-  s.invZ = fp; fp += R;
-  s.m = fp; fp += R;
   s.rowm = fp; fp += R;
   s.rows = fp; fp += R;
   s.dbgp = fp; fp += R;
   s.mask_val = fp; fp += R;
-  int nt = (V + kTile - 1) / kTile;
+  const int nt = (V + kTile - 1) / kTile;
   s.tsum = fp; fp += nt;
   s.tmax = fp; fp += nt;
   s.state = reinterpret_cast<uint8_t*>(fp);
@@ -223,8 +244,8 @@ __device__ __forceinline__ TravSmem carve(char* base, int R, int V) {
 struct Control {
   // serial state of the traversal, owned by thread 0
   int node = 0;
-  int pending = -1;      // child whose rejection the running pass serves
-  float masked_sum = 0;  // sum of m over the removed tokens of that pass
+  int pending = -1;       // child whose rejection the running pass serves
+  double masked_sum = 0;  // sum of m over the removed tokens of that pass
   int n_tests = 0, n_passes = 0;
 };
 
@@ -234,41 +255,42 @@ __device__ __forceinline__ int first_alive_child(const TravSmem& s, int i) {
   return j;
 }
 
-// M_b^(0)(x_c | parent) from the gathered logit of the child's token.
-__device__ __forceinline__ float mb0_of(const TravSmem& s, int i, int c, float cT) {
-  return ex2((s.gl[c] - s.rowm[i]) * cT) / s.rows[i];
+// M_b^(0)(x_c | X^i) of child c's token.  The numerator is evaluated in
+// float64: a residual a M_b(x) - b M_s(x) formed from it can cancel by orders
+// of magnitude, and a single float32 exponential (unlike the row sum, which
+// averages many) would carry its full rounding into the child's rate.
+__device__ __forceinline__ double mb0_of(const TravSmem& s, int i, int c, double cd) {
+  return exp2(((double)s.gl[c] - (double)s.rowm[i]) * cd) / (double)s.rows[i];
 }
 
 // Rate of child c of node i from i's current state:
-// min(p_i * M_b(x_c) / M_s(x_c), 1).  Returns false if M_s(x_c) == 0.
-__device__ __forceinline__ bool child_rate(const TravSmem& s, int i, int c, float cT, float* out) {
-  float mb = fmaxf(fmaf(s.a[i], mb0_of(s, i, c, cT), -s.b[i] * s.gq[c]), 0.f);
-  float ms = s.gq[c] * s.invZ[i];
-  if (!(ms > 0.f)) return false;
-  float r = s.p[i] * mb / ms;
-  *out = fminf(r, 1.f);
+// min(p_i M_b(x_c) / M_s(x_c), 1).  Returns false if M_s(x_c) == 0.
+__device__ __forceinline__ bool child_rate(const TravSmem& s, int i, int c, double cd, double* out) {
+  const double q = (double)s.gq[c];
+  const double mb = fmax(s.a[i] * mb0_of(s, i, c, cd) - s.b[i] * q, 0.0);
+  const double ms = q * s.invZ[i];
+  if (!(ms > 0.0)) return false;
+  *out = fmin(s.p[i] * mb / ms, 1.0);
   return true;
 }
 
 __device__ void start_pass(const TravSmem& s, Ctl& ctl, Control& st, int i, int c) {
   st.pending = c;
-  const float p = s.p[i];
-  ctl.alpha1 = p * s.a[i] / s.rows[i];
-  ctl.beta = fmaf(p, s.b[i], s.invZ[i]);
+  const double p = s.p[i];
+  ctl.alpha1 = (float)(p * s.a[i] / (double)s.rows[i]);
+  ctl.beta = (float)(p * s.b[i] + s.invZ[i]);
   int n = 0;
-  float msum = 0.f;
+  double msum = 0.0;
   for (int j = s.first[i]; j >= 0; j = s.next[j]) {
     if (j == c || s.state[j] == kAlive) continue;
-    // insert the removed token in increasing order
-    int t = s.tok[j];
+    // removed tokens in increasing order
+    const int t = s.tok[j];
     int k = n;
     while (k > 0 && s.mask_tok[k - 1] > t) {
       s.mask_tok[k] = s.mask_tok[k - 1];
-      s.mask_val[k] = s.mask_val[k - 1];
       --k;
     }
     s.mask_tok[k] = t;
-    s.mask_val[k] = s.m[j];
     msum += s.m[j];
     ++n;
   }
@@ -281,42 +303,42 @@ __device__ void start_pass(const TravSmem& s, Ctl& ctl, Control& st, int i, int 
 }
 
 // Eqs. (1)-(3) at node i after removing child c, in the (a, b, Z) form.
-__device__ void apply_rejection(const TravSmem& s, Ctl& ctl, Control& st, int i, int c, float cT) {
-  const float p = s.p[i], a = s.a[i], b = s.b[i];
-  const float S = ctl.S + p * st.masked_sum;
-  const float alpha = p * a;
-  const float beta = fmaf(p, b, s.invZ[i]);
-  const float mb0 = mb0_of(s, i, c, cT);
-  const float q0 = s.gq[c];
-  if (S > 0.f) {
-    const float na = alpha / S, nb = beta / S, scale = p / S;
+__device__ void apply_rejection(const TravSmem& s, Ctl& ctl, Control& st, int i, int c, double cd) {
+  const double p = s.p[i], a = s.a[i], b = s.b[i];
+  const double S = (double)ctl.S + p * st.masked_sum;
+  const double alpha = p * a;
+  const double beta = p * b + s.invZ[i];
+  const double mb0 = mb0_of(s, i, c, cd);
+  const double q0 = (double)s.gq[c];
+  if (S > 0.0) {
+    const double na = alpha / S, nb = beta / S, scale = p / S;
     for (int j = s.first[i]; j >= 0; j = s.next[j])
       if (j != c && s.state[j] != kAlive) s.m[j] *= scale;
-    s.m[c] = fmaxf(fmaf(na, mb0, -nb * q0), 0.f);
+    s.m[c] = fmax(na * mb0 - nb * q0, 0.0);
     s.a[i] = na;
     s.b[i] = nb;
-    s.p[i] = S / (S + (1.f - p));
+    s.p[i] = S / (S + (1.0 - p));
   } else {
     // 0/0 in Eqs. (1)/(3): the node keeps its target distribution; its rate
     // becomes 0 (it can no longer be accepted) unless it was 1.
     ctl.bad |= 16u;
-    s.m[c] = fmaxf(fmaf(a, mb0, -b * q0), 0.f);
-    s.p[i] = (p == 1.f) ? 1.f : 0.f;
+    s.m[c] = fmax(a * mb0 - b * q0, 0.0);
+    s.p[i] = (p == 1.0) ? 1.0 : 0.0;
   }
-  const float Z = s.Z[i] - q0;
+  const double Z = s.Z[i] - q0;
   s.Z[i] = Z;
-  s.invZ[i] = (Z > 0.f) ? 1.f / Z : 0.f;
+  s.invZ[i] = (Z > 0.0) ? 1.0 / Z : 0.0;
 }
 
 // Runs the serial traversal until a vocabulary pass is needed or it ends.
 __device__ void control_step(const TravSmem& s, Ctl& ctl, Control& st, const float* __restrict__ u,
-                             float cT) {
+                             double cd) {
   if (st.pending >= 0) {
     const int c = st.pending, i = s.par[c];
-    apply_rejection(s, ctl, st, i, c, cT);
+    apply_rejection(s, ctl, st, i, c, cd);
     st.pending = -1;
     st.node = i;
-    if (i != 0 && s.p[i] == 0.f) {   // rate 0: remove i with what is left below it
+    if (i != 0 && s.p[i] == 0.0) {   // rate 0: remove i with what is left below it
       s.state[i] = kPruned;
       s.dbgp[i] = 0.f;
       start_pass(s, ctl, st, s.par[i], i);
@@ -329,20 +351,20 @@ __device__ void control_step(const TravSmem& s, Ctl& ctl, Control& st, const flo
     if (c < 0) {
       if (node == 0) { ctl.accepted = 0; ctl.cmd = kCmdDone; return; }
       st.n_tests++;
-      s.dbgp[node] = s.p[node];
-      if (u[node] < s.p[node]) { ctl.accepted = node; ctl.cmd = kCmdDone; return; }
+      s.dbgp[node] = (float)s.p[node];
+      if ((double)u[node] < s.p[node]) { ctl.accepted = node; ctl.cmd = kCmdDone; return; }
       s.state[node] = kRejected;
       start_pass(s, ctl, st, s.par[node], node);
       return;
     }
-    float pc;
-    if (!child_rate(s, node, c, cT, &pc)) {
+    double pc;
+    if (!child_rate(s, node, c, cd, &pc)) {
       ctl.bad |= 8u;
       ctl.accepted = -1;
       ctl.cmd = kCmdDone;
       return;
     }
-    if (pc == 0.f) {
+    if (pc == 0.0) {
       s.state[c] = kPruned;
       s.dbgp[c] = 0.f;
       start_pass(s, ctl, st, node, c);
@@ -361,7 +383,7 @@ __global__ void __launch_bounds__(kTravThreads, 1) tv_traverse_kernel(TravArgs a
   const int R = args.N + 1, V = args.V;
   const int b = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
-  const float cT = args.cT;
+  const float c_hi = args.c_hi, c_lo = args.c_lo;
   TravSmem s = carve(smem_raw, R, V);
   const typename L::elem* logits = reinterpret_cast<const typename L::elem*>(args.logits);
   const size_t tree_row0 = (size_t)b * R;
@@ -377,12 +399,12 @@ __global__ void __launch_bounds__(kTravThreads, 1) tv_traverse_kernel(TravArgs a
     s.first[i] = 0x7fffffff;
     s.npass[i] = 0;
     s.state[i] = kAlive;
-    s.a[i] = 1.f;
-    s.b[i] = 0.f;
-    s.Z[i] = 1.f;
-    s.invZ[i] = 1.f;
-    s.m[i] = 0.f;
-    s.p[i] = 0.f;
+    s.a[i] = 1.0;
+    s.b[i] = 0.0;
+    s.Z[i] = 1.0;
+    s.invZ[i] = 1.0;
+    s.m[i] = 0.0;
+    s.p[i] = 0.0;
     s.dbgp[i] = __int_as_float(0x7fc00000);
   }
   __syncthreads();
@@ -435,7 +457,7 @@ __global__ void __launch_bounds__(kTravThreads, 1) tv_traverse_kernel(TravArgs a
         s.rows[i] = st2.y;
       }
     }
-    if (tid == 0) s.p[0] = 1.f;
+    if (tid == 0) s.p[0] = 1.0;
   }
   __syncthreads();
 
@@ -443,7 +465,7 @@ __global__ void __launch_bounds__(kTravThreads, 1) tv_traverse_kernel(TravArgs a
   const float* u = args.uniforms + (size_t)b * (R + 1);
   if (ok) {
     for (;;) {
-      if (tid == 0) control_step(s, ctl, st, u, cT);
+      if (tid == 0) control_step(s, ctl, st, u, args.c);
       __syncthreads();
       if (ctl.cmd == kCmdDone) break;
       // ---- S = sum over tokens not removed of [alpha1 e(x) - beta q(x)]_+ ----
@@ -459,7 +481,8 @@ __global__ void __launch_bounds__(kTravThreads, 1) tv_traverse_kernel(TravArgs a
         load_logits<L, VEC>(lrow, x0, V, v);
         load_probs<VEC>(qrow, x0, V, q);
 #pragma unroll
-        for (int k = 0; k < 8; ++k) t[k] = fmaxf(fmaf(al, ex2((v[k] - m) * cT), -be * q[k]), 0.f);
+        for (int k = 0; k < 8; ++k)
+          t[k] = fmaxf(fmaf(al, L::exp_rel(v[k], m, c_hi, c_lo), -be * q[k]), 0.f);
         while (mp < nmask && s.mask_tok[mp] < x0) ++mp;
         for (int mq = mp; mq < nmask && s.mask_tok[mq] < x0 + kChunk; ++mq) {
           const int off = s.mask_tok[mq] - x0;
@@ -501,21 +524,20 @@ __global__ void __launch_bounds__(kTravThreads, 1) tv_traverse_kernel(TravArgs a
             --k;
           }
           s.mask_tok[k] = t;
-          s.mask_val[k] = s.m[j];
+          s.mask_val[k] = (float)s.m[j];
           ++n;
         }
-        ctl.bonus_a = s.a[a] / s.rows[a];
-        ctl.bonus_b = s.b[a];
+        ctl.bonus_a = (float)(s.a[a] / (double)s.rows[a]);
+        ctl.bonus_b = (float)s.b[a];
         ctl.rowmax = s.rowm[a];
       }
       ctl.nmask = n;
-      ctl.bonus_leaf = leaf ? 1 : 0;
     }
     __syncthreads();
     const int nt = (V + kTile - 1) / kTile;
     const int nmask = ctl.nmask;
     const float ba = ctl.bonus_a, bb = ctl.bonus_b, rm = ctl.rowmax;
-    // pass 1: per warp-tile sums (leaf: with the tile's own max)
+    // pass 1: per warp-tile sums (leaf: relative to the tile's own max)
     int mp = 0;
     for (int k = wid; k < nt; k += kTravWarps) {
       const int x0 = k * kTile + lane * kChunk;
@@ -532,7 +554,8 @@ __global__ void __launch_bounds__(kTravThreads, 1) tv_traverse_kernel(TravArgs a
         for (int e = 1; e < 8; ++e) lm = fmaxf(lm, v[e]);
         const float tm = warp_max(lm);
 #pragma unroll
-        for (int e = 0; e < 8; ++e) w[e] = (v[e] == TV_NEG_INF) ? 0.f : ex2((v[e] - tm) * cT);
+        for (int e = 0; e < 8; ++e)
+          w[e] = (v[e] == TV_NEG_INF) ? 0.f : L::exp_rel(v[e], tm, c_hi, c_lo);
         const float ts = warp_sum(sum8(w));
         if (lane == 0) { s.tsum[k] = ts; s.tmax[k] = tm; }
       } else {
@@ -545,7 +568,9 @@ __global__ void __launch_bounds__(kTravThreads, 1) tv_traverse_kernel(TravArgs a
           for (int e = 0; e < 8; ++e) { v[e] = TV_NEG_INF; q[e] = 0.f; }
         }
 #pragma unroll
-        for (int e = 0; e < 8; ++e) w[e] = fmaxf(fmaf(ba, ex2((v[e] - rm) * cT), -bb * q[e]), 0.f);
+        for (int e = 0; e < 8; ++e)
+          w[e] = (v[e] == TV_NEG_INF) ? 0.f
+                                      : fmaxf(fmaf(ba, L::exp_rel(v[e], rm, c_hi, c_lo), -bb * q[e]), 0.f);
         while (mp < nmask && s.mask_tok[mp] < x0) ++mp;
         for (int mq = mp; mq < nmask && s.mask_tok[mq] < x0 + kChunk; ++mq) {
           const int off = s.mask_tok[mq] - x0;
@@ -566,7 +591,7 @@ __global__ void __launch_bounds__(kTravThreads, 1) tv_traverse_kernel(TravArgs a
         for (int k = lane; k < nt; k += 32) lm = fmaxf(lm, s.tmax[k]);
         M = warp_max(lm);
         for (int k = lane; k < nt; k += 32)
-          s.tsum[k] = (s.tmax[k] == TV_NEG_INF) ? 0.f : s.tsum[k] * ex2((s.tmax[k] - M) * cT);
+          s.tsum[k] = (s.tmax[k] == TV_NEG_INF) ? 0.f : s.tsum[k] * L::exp_rel(s.tmax[k], M, c_hi, c_lo);
         __syncwarp();
       }
       float base = 0.f;
@@ -618,7 +643,8 @@ __global__ void __launch_bounds__(kTravThreads, 1) tv_traverse_kernel(TravArgs a
           for (int e = 0; e < 8; ++e) v[e] = TV_NEG_INF;
         }
 #pragma unroll
-        for (int e = 0; e < 8; ++e) w[e] = (v[e] == TV_NEG_INF) ? 0.f : ex2((v[e] - M) * cT);
+        for (int e = 0; e < 8; ++e)
+          w[e] = (v[e] == TV_NEG_INF) ? 0.f : L::exp_rel(v[e], M, c_hi, c_lo);
       } else {
         float v[8], q[8];
         if (x0 < V) {
@@ -629,7 +655,9 @@ __global__ void __launch_bounds__(kTravThreads, 1) tv_traverse_kernel(TravArgs a
           for (int e = 0; e < 8; ++e) { v[e] = TV_NEG_INF; q[e] = 0.f; }
         }
 #pragma unroll
-        for (int e = 0; e < 8; ++e) w[e] = fmaxf(fmaf(ba, ex2((v[e] - rm) * cT), -bb * q[e]), 0.f);
+        for (int e = 0; e < 8; ++e)
+          w[e] = (v[e] == TV_NEG_INF) ? 0.f
+                                      : fmaxf(fmaf(ba, L::exp_rel(v[e], rm, c_hi, c_lo), -bb * q[e]), 0.f);
         for (int mq = 0; mq < nmask; ++mq) {
           const int off = s.mask_tok[mq] - x0;
           const float mv = s.mask_val[mq];
@@ -669,10 +697,10 @@ __global__ void __launch_bounds__(kTravThreads, 1) tv_traverse_kernel(TravArgs a
           yy = V - 1;
         }
       }
-      if (lane == 0) { ctl.W = W; ctl.bonus_tile = yy; }
+      if (lane == 0) ctl.bonus_y = yy;
     }
     __syncthreads();
-    y = ctl.bonus_tile;
+    y = ctl.bonus_y;
   }
 
   // ---- outputs ----
@@ -719,8 +747,8 @@ int launch_error() {
 }  // namespace
 
 size_t tv_traverse_smem_bytes(int R, int V) {
-  int nt = (V + tvk::kTile - 1) / tvk::kTile;
-  return (size_t)R * (6 * 4 + 14 * 4 + 1) + (size_t)nt * 8 + 64;
+  const int nt = (V + tvk::kTile - 1) / tvk::kTile;
+  return (size_t)R * (6 * 8 + 6 * 4 + 6 * 4 + 1) + (size_t)nt * 8 + 64;
 }
 
 namespace {
@@ -738,7 +766,7 @@ int launch_typed(const TravArgs& a, int* row_list, int* n_rows, int stats_grid,
   if (launch_error()) return -5;
   if (ev && cudaEventRecord(ev[1], stream) != cudaSuccess) return -5;
   tvk::tv_row_stats_kernel<L, VEC><<<stats_grid, tvk::kStatsThreads, 0, stream>>>(
-      lg, a.V, a.cT, row_list, n_rows, a.stats);
+      lg, a.V, a.c_hi, a.c_lo, row_list, n_rows, a.stats);
   if (launch_error()) return -5;
   if (ev && cudaEventRecord(ev[2], stream) != cudaSuccess) return -5;
   if (cudaFuncSetAttribute(tvk::tv_traverse_kernel<L, VEC>,

@@ -13,7 +13,8 @@ struct TravArgs {
   const float* uniforms;       // [B][N+2]
   float2* stats;               // [B][N+1] row (max, sum of exp2) of internal rows
   int B, N, V;
-  float cT;                    // log2(e) / temperature
+  float c_hi, c_lo;            // log2(e) / temperature = c_hi + c_lo
+  double c;                    // the same constant in float64
   int32_t* out_path;           // [B][N]
   int32_t* out_accept_len;     // [B]
   int32_t* out_bonus;          // [B]

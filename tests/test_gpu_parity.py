@@ -43,7 +43,8 @@ def check(tv, inp, trees=None, max_tie_frac=0.25):
     det = {trees[k]: r for k, r in det.items()}
     summ = compare_batch(det, path, tau, bonus, node_p, stats)
     print(f"\n{inp.meta}: trees {summ['trees']} exact {summ['exact']} "
-          f"ties {summ['ties']} max p rel err {summ['max_p_rel']:.2e}")
+          f"ties {summ['ties']} max p rel err {summ['max_p_rel']:.2e} "
+          f"ill-conditioned {summ['ill']} (max kappa {summ['max_kappa']:.3g})")
     assert not summ["bad"], summ["bad"][:5]
     assert summ["ties"] <= max_tie_frac * summ["trees"] + 1
     return summ, status

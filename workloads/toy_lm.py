@@ -104,3 +104,69 @@ def sample_draft_trees(parents, ms_table, vocab, count, seed, with_replacement=F
             pre.append(pre[par] + (x,))
         out[b] = toks
     return out
+
+
+def prefix_code(prefix, vocab):
+    """Integer code of a prefix: root 0, child code = parent * (V + 1) + x + 1."""
+    c = 0
+    for x in prefix:
+        c = c * (vocab + 1) + x + 1
+    return c
+
+
+def table_array(table, vocab, max_len):
+    """Dense [(V+1)^(max_len+1), V] float64 array of a float table, indexed by
+    prefix_code (unused codes hold zeros)."""
+    out = np.zeros(((vocab + 1) ** (max_len + 1), vocab))
+    for pre, row in table.items():
+        out[prefix_code(pre, vocab)] = np.asarray(row, dtype=np.float64)
+    return out
+
+
+def sample_trees_batch(parents, ms_array, vocab, count, rng):
+    """Vectorised draw of ``count`` draft trees of one shape (Definition 1,
+    children without replacement in index order) from a dense table array.
+    Returns (tokens [count, N+1] int64, prefix codes [count, N+1] int64)."""
+    n = len(parents)
+    tokens = np.zeros((count, n), dtype=np.int64)
+    codes = np.zeros((count, n), dtype=np.int64)
+    rows = np.arange(count)
+    for i in range(1, n):
+        par = parents[i]
+        probs = ms_array[codes[:, par]].copy()
+        for j in range(1, i):
+            if parents[j] == par:
+                probs[rows, tokens[:, j]] = 0.0
+        probs /= probs.sum(axis=1, keepdims=True)
+        cdf = np.cumsum(probs, axis=1)
+        u = rng.random(count)[:, None]
+        x = np.minimum((u >= cdf).sum(axis=1), vocab - 1)
+        # never land on a zero-probability token through rounding
+        bad = probs[rows, x] == 0
+        while bad.any():
+            x[bad] = np.argmax(probs[bad] > 0, axis=1)
+            bad = probs[rows, x] == 0
+        tokens[:, i] = x
+        codes[:, i] = codes[:, par] * (vocab + 1) + x + 1
+    return tokens, codes
+
+
+def extend_with_target(first_tokens, mb_array, vocab, length, rng):
+    """Complete sequences to ``length`` tokens by sampling the target table:
+    ``first_tokens`` is a list (per sample) of the tokens already fixed."""
+    count = len(first_tokens)
+    out = np.full((count, length), -1, dtype=np.int64)
+    code = np.zeros(count, dtype=np.int64)
+    for b, toks in enumerate(first_tokens):
+        for j, x in enumerate(toks[:length]):
+            out[b, j] = x
+    for j in range(length):
+        need = out[:, j] < 0
+        if need.any():
+            probs = mb_array[code[need]]
+            cdf = np.cumsum(probs, axis=1)
+            u = rng.random(int(need.sum()))[:, None] * cdf[:, -1:]
+            x = np.minimum((u >= cdf).sum(axis=1), vocab - 1)
+            out[need, j] = x
+        code = code * (vocab + 1) + out[:, j] + 1
+    return out
