@@ -215,6 +215,7 @@ def main():
                                      inp.temperature, inp.uniforms, debug=True)
     torch.cuda.synchronize(dev)
     row_bytes, trav_bytes = algorithmic_bytes(inp.parents, stats, V, lb)
+    fused, cluster, warps, stages = v.launch_shape(B, N)
     a_bytes = row_bytes + trav_bytes
     mean_tau1 = float(tau_d.float().mean()) + 1.0
     passes_per_tree = float(stats[:, 1].float().mean())
@@ -329,7 +330,9 @@ def main():
                    "logit_dtype": "bf16" if lb == 2 else "fp32",
                    "temperature": w.temperature, "sigma": w.sigma, "seed": args.seed,
                    "l2": "flushed by a 256 MiB write before every timed step (untimed)",
-                   "parallelism": f"dp{world} (independent trees per GPU)"},
+                   "parallelism": f"dp{world} (independent trees per GPU)",
+                   "kernel_path": "fused" if fused else "three-kernel",
+                   "ctas_per_tree": cluster, "consumer_warps": warps, "ring_stages": stages},
         "verified_logit_gbps": round(step_gbs, 2),
         "hbm_frac_step": round(step_gbs / peak, 4),
         "algorithmic_bytes_per_step": a_bytes,

@@ -62,12 +62,23 @@ enum {
                                   draws children without replacement) */
   TV_STATUS_ZERO_DRAFT = 8u,   /* a drafted token has zero draft probability at its
                                   parent, so it cannot have come from M_s */
-  TV_STATUS_DEGENERATE = 16u   /* informational: S = 0 occurred in Eqs. (1)/(3); the
+  TV_STATUS_DEGENERATE = 16u,  /* informational: S = 0 occurred in Eqs. (1)/(3); the
                                   0/0 was resolved as p' = 0 (p < 1) or p' = 1 (p = 1) */
+  TV_STATUS_TIMEOUT = 32u,     /* a bounded device wait gave up (not expected; the tree's
+                                  outputs are -1) */
+  TV_STATUS_BAD_ROW = 64u      /* a target row the traversal needed has no finite logit */
 };
 
 /* Flags for tv_create. */
-enum { TV_FLAG_NONE = 0u };
+enum {
+  TV_FLAG_NONE = 0u,
+  /* Use the three-kernel path (row normalisers of every internal row, then one
+     CTA per tree) even when the fused single-kernel path is available.  The
+     fused path (one thread-block cluster per tree, rows read lazily through
+     bulk copies) needs V % 8 == 0; other vocabularies always take the
+     three-kernel path.  Both compute the same results. */
+  TV_FLAG_UNFUSED = 1u
+};
 
 /*
  * tv_create -- allocate a handle and its device workspace.
@@ -78,7 +89,7 @@ enum { TV_FLAG_NONE = 0u };
  *                may pass; 0 <= max_nodes <= 1023.
  *   max_batch  : largest B later calls may pass; >= 1.
  *   logit_dtype: element type of target_logits in later calls.
- *   flags      : TV_FLAG_NONE.
+ *   flags      : TV_FLAG_NONE or TV_FLAG_UNFUSED.
  * Errors: TV_ERR_INVALID_ARG, TV_ERR_VOCAB, TV_ERR_CUDA, TV_ERR_DEVICE.
  */
 int tv_create(tv_handle** out, int device, int vocab, int max_nodes, int max_batch,
@@ -182,6 +193,16 @@ int tv_set_phase_timing(tv_handle* h, int enable);
  * (timing off or no timed call yet), TV_ERR_CUDA.
  */
 int tv_last_phase_ms(tv_handle* h, float* ms);
+
+/*
+ * tv_launch_shape -- how a call with these B and N would run on this handle:
+ * *path = 1 for the fused single-kernel path, 0 for the three-kernel path;
+ * for the fused path also the thread-block cluster size (CTAs per tree), the
+ * consumer warps per CTA and the ring stages.  Any output pointer may be NULL.
+ * Errors: TV_ERR_INVALID_ARG, TV_ERR_CAPACITY.
+ */
+int tv_launch_shape(tv_handle* h, int B, int N, int* path, int* cluster, int* warps,
+                    int* stages);
 
 /* tv_destroy -- free the handle's workspace (synchronises its device). */
 int tv_destroy(tv_handle* h);

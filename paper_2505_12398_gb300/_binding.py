@@ -13,6 +13,8 @@ TV_STATUS = {
     "DUP_SIBLING": 4,
     "ZERO_DRAFT": 8,
     "DEGENERATE": 16,
+    "TIMEOUT": 32,
+    "BAD_ROW": 64,
 }
 
 
@@ -44,6 +46,8 @@ _SIGS = {
     "tv_destroy": (_I, [_P]),
     "tv_set_phase_timing": (_I, [_P, _I]),
     "tv_last_phase_ms": (_I, [_P, ctypes.POINTER(ctypes.c_float)]),
+    "tv_launch_shape": (_I, [_P, _I, _I, ctypes.POINTER(_I), ctypes.POINTER(_I),
+                             ctypes.POINTER(_I), ctypes.POINTER(_I)]),
     "tv_strerror": (ctypes.c_char_p, [_I]),
     "tv_version": (_I, []),
 }
@@ -89,7 +93,7 @@ class Verifier:
     the handle's device with the dtypes and layouts of include/tv.h.
     """
 
-    def __init__(self, vocab, max_nodes, max_batch, logit_dtype="bf16", device=0):
+    def __init__(self, vocab, max_nodes, max_batch, logit_dtype="bf16", device=0, unfused=False):
         import torch
         self.lib = library()
         if logit_dtype in ("bf16", torch.bfloat16, TV_BF16):
@@ -102,7 +106,7 @@ class Verifier:
         self.device = torch.device("cuda", device) if isinstance(device, int) else torch.device(device)
         h = ctypes.c_void_p()
         rc = self.lib.tv_create(ctypes.byref(h), self.device.index or 0, vocab, max_nodes,
-                                max_batch, self.dtype_code, 0)
+                                max_batch, self.dtype_code, 1 if unfused else 0)
         if rc != 0:
             raise LibraryError("tv_create", rc, self.lib)
         self.handle = h
@@ -195,6 +199,14 @@ class Verifier:
         if rc != 0:
             raise LibraryError("tv_last_phase_ms", rc, self.lib)
         return [float(x) for x in ms]
+
+    def launch_shape(self, B, N):
+        """(fused path?, CTAs per tree, consumer warps per CTA, ring stages)."""
+        out = [ctypes.c_int() for _ in range(4)]
+        rc = self.lib.tv_launch_shape(self.handle, B, N, *[ctypes.byref(o) for o in out])
+        if rc != 0:
+            raise LibraryError("tv_launch_shape", rc, self.lib)
+        return tuple(o.value for o in out)
 
     def status(self):
         """Synchronise and return (and clear) the TV_STATUS_* bits raised."""

@@ -6,6 +6,7 @@
 
 #include <cmath>
 #include <cstdint>
+#include <cstdio>
 #include <cstdlib>
 #include <new>
 
@@ -20,6 +21,9 @@ struct tv_handle {
   tv_dtype dtype = TV_BF16;
   unsigned flags = 0;
   int sm_count = 0;
+  int smem_per_sm = 0;
+  int smem_per_block = 0;
+  int force_ncw = 0, force_c = 0, force_stages = 0;   // tuning override (TV_FUSED_PLAN)
   // device workspace
   int32_t* row_list = nullptr;   // [max_batch * (max_nodes + 1)]
   int32_t* n_rows = nullptr;     // [1]
@@ -110,8 +114,18 @@ int verify_impl(tv_handle* h, int B, int N, const int32_t* parents, const int32_
   int grid = h->sm_count * 4;
   if (grid > rows) grid = rows;
   if (grid < 1) grid = 1;
-  rc = tv_launch_all(a, h->dtype == TV_BF16 ? 1 : 0, h->row_list, h->n_rows, grid,
-                     static_cast<cudaStream_t>(stream), h->timing ? h->ev : nullptr);
+  const bool fused = (h->vocab % 8) == 0 && !(h->flags & TV_FLAG_UNFUSED);
+  FusedPlan plan;
+  if (fused)
+    plan = tv_fused_plan(B, N + 1, h->vocab, h->sm_count, h->smem_per_sm, h->smem_per_block,
+                         h->force_ncw, h->force_c, h->force_stages);
+  if (fused && plan.ok) {
+    rc = tv_launch_fused(a, h->dtype == TV_BF16 ? 1 : 0, plan, static_cast<cudaStream_t>(stream),
+                         h->timing ? h->ev : nullptr);
+  } else {
+    rc = tv_launch_all(a, h->dtype == TV_BF16 ? 1 : 0, h->row_list, h->n_rows, grid,
+                       static_cast<cudaStream_t>(stream), h->timing ? h->ev : nullptr);
+  }
   if (rc == TV_OK && h->timing) h->timed_call = true;
   return rc;
 }
@@ -127,7 +141,7 @@ int tv_create(tv_handle** out, int device, int vocab, int max_nodes, int max_bat
   if (vocab < 1 || vocab > kMaxVocab) return TV_ERR_VOCAB;
   if (max_nodes < 0 || max_nodes + 1 > kMaxRows || max_batch < 1) return TV_ERR_INVALID_ARG;
   if (logit_dtype != TV_BF16 && logit_dtype != TV_FP32) return TV_ERR_INVALID_ARG;
-  if (flags != TV_FLAG_NONE) return TV_ERR_INVALID_ARG;
+  if (flags & ~TV_FLAG_UNFUSED) return TV_ERR_INVALID_ARG;
   int ndev = 0;
   if (cudaGetDeviceCount(&ndev) != cudaSuccess || device < 0 || device >= ndev) {
     cudaGetLastError();
@@ -148,6 +162,12 @@ int tv_create(tv_handle** out, int device, int vocab, int max_nodes, int max_bat
   h->dtype = logit_dtype;
   h->flags = flags;
   h->sm_count = prop.multiProcessorCount;
+  h->smem_per_sm = (int)prop.sharedMemPerMultiprocessor;
+  h->smem_per_block = (int)prop.sharedMemPerBlockOptin;
+  // TV_FUSED_PLAN="ncw,cluster,stages" overrides the fused kernel's launch
+  // shape (tuning only; invalid values are ignored)
+  if (const char* env = std::getenv("TV_FUSED_PLAN"))
+    std::sscanf(env, "%d,%d,%d", &h->force_ncw, &h->force_c, &h->force_stages);
   DeviceGuard guard(device);
   if (!guard.ok()) {
     delete h;
@@ -304,6 +324,23 @@ int tv_last_phase_ms(tv_handle* h, float* ms) {
       return TV_ERR_CUDA;
     }
   }
+  return TV_OK;
+}
+
+int tv_launch_shape(tv_handle* h, int B, int N, int* path, int* cluster, int* warps,
+                    int* stages) {
+  if (!h || B < 0 || N < 0) return TV_ERR_INVALID_ARG;
+  if (B > h->max_batch || N > h->max_nodes) return TV_ERR_CAPACITY;
+  const bool fused = (h->vocab % 8) == 0 && !(h->flags & TV_FLAG_UNFUSED);
+  FusedPlan plan;
+  if (fused)
+    plan = tv_fused_plan(B, N + 1, h->vocab, h->sm_count, h->smem_per_sm, h->smem_per_block,
+                         h->force_ncw, h->force_c, h->force_stages);
+  const bool f = fused && plan.ok;
+  if (path) *path = f ? 1 : 0;
+  if (cluster) *cluster = f ? plan.C : 1;
+  if (warps) *warps = f ? plan.ncw : 16;
+  if (stages) *stages = f ? plan.stages : 0;
   return TV_OK;
 }
 

@@ -448,13 +448,14 @@ __global__ void __launch_bounds__(kTravThreads, 1) tv_traverse_kernel(TravArgs a
     if (bad) atomicOr(&ctl.bad, bad);
   }
   __syncthreads();
-  const bool ok = (ctl.bad == 0u);
+  bool ok = (ctl.bad == 0u);
   if (ok) {
     for (int i = tid; i < R; i += kTravThreads) {
       if (s.first[i] >= 0) {
         const float2 st2 = args.stats[tree_row0 + i];
         s.rowm[i] = st2.x;
         s.rows[i] = st2.y;
+        if (!(st2.y > 0.f)) atomicOr(&ctl.bad, 64u);   // no finite logit in the row
       }
     }
     if (tid == 0) s.p[0] = 1.0;
@@ -463,6 +464,7 @@ __global__ void __launch_bounds__(kTravThreads, 1) tv_traverse_kernel(TravArgs a
 
   Control st;
   const float* u = args.uniforms + (size_t)b * (R + 1);
+  if (ok && (ctl.bad & 64u)) ok = false;
   if (ok) {
     for (;;) {
       if (tid == 0) control_step(s, ctl, st, u, args.c);

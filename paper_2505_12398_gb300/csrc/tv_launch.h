@@ -23,6 +23,24 @@ struct TravArgs {
   uint32_t* status;            // status word (OR of TV_STATUS_* bits)
 };
 
+// Launch plan of the fused kernel: cluster size, ring stages, shared memory.
+struct FusedPlan {
+  int ncw = 8;       // consumer warps per CTA (4 or 8)
+  int C = 1;
+  int stages = 0;
+  size_t smem = 0;
+  bool ok = false;
+};
+
+FusedPlan tv_fused_plan(int B, int R, int V, int sm_count, int smem_per_sm, int smem_per_block,
+                        int force_ncw, int force_c, int force_stages);
+
+// Queues the fused kernel (one cluster of plan.C CTAs per tree).  Requires
+// V % 8 == 0 (16-byte aligned rows for the bulk copies).  With `events`,
+// events[0..2] are recorded before and events[3] after it.
+int tv_launch_fused(const TravArgs& a, int logit_is_bf16, const FusedPlan& plan,
+                    cudaStream_t stream, cudaEvent_t* events);
+
 // Dynamic shared memory the traversal kernel needs for R = N+1 rows.
 size_t tv_traverse_smem_bytes(int R, int V);
 

@@ -21,11 +21,11 @@ def tv():
     return tv
 
 
-def run_gpu(tv, inp, debug=True):
+def run_gpu(tv, inp, debug=True, unfused=False):
     B, R = inp.parents.shape
     V = inp.logits.shape[-1]
     dt = "bf16" if inp.logits.dtype == torch.bfloat16 else "fp32"
-    v = tv.Verifier(V, R - 1, B, dt)
+    v = tv.Verifier(V, R - 1, B, dt, unfused=unfused)
     out = v.verify(inp.parents, inp.tokens, inp.logits, inp.draft_probs, inp.temperature,
                    inp.uniforms, debug=debug)
     torch.cuda.synchronize()
@@ -34,8 +34,8 @@ def run_gpu(tv, inp, debug=True):
     return [o.cpu().numpy() for o in out], status
 
 
-def check(tv, inp, trees=None, max_tie_frac=0.25):
-    (path, tau, bonus, node_p, stats), status = run_gpu(tv, inp)
+def check(tv, inp, trees=None, max_tie_frac=0.25, unfused=False):
+    (path, tau, bonus, node_p, stats), status = run_gpu(tv, inp, unfused=unfused)
     if trees is None:
         trees = list(range(inp.parents.shape[0]))
     par, tok, lg, dp, un = to_numpy_inputs(inp, trees)
@@ -50,11 +50,12 @@ def check(tv, inp, trees=None, max_tie_frac=0.25):
     return summ, status
 
 
-def test_tiny_many_seeds(tv):
+@pytest.mark.parametrize("unfused", [False, True])
+def test_tiny_many_seeds(tv, unfused):
     """The 7-node, V=64, fp32 tree, 512 draws of logits / tree / uniforms."""
     w = get_workload("tiny", batch=512)
     inp = make_inputs(w, seed=0, device="cuda")
-    summ, status = check(tv, inp)
+    summ, status = check(tv, inp, unfused=unfused)
     assert summ["exact"] >= 0.9 * summ["trees"]
     assert status & ~16 == 0
 
@@ -67,18 +68,45 @@ def test_chain_and_binary(tv, name, sigma):
     check(tv, inp)
 
 
-def test_eagle_v32k_all_trees(tv):
+@pytest.mark.parametrize("unfused", [False, True])
+def test_eagle_v32k_all_trees(tv, unfused):
     w = get_workload("eagle_v32k")
     inp = make_inputs(w, seed=2, device="cuda")
-    check(tv, inp)
+    check(tv, inp, unfused=unfused)
 
 
-def test_eagle_v128k_sampled(tv):
+@pytest.mark.parametrize("unfused", [False, True])
+def test_eagle_v128k_sampled(tv, unfused):
     """Full batch of 128 trees at V=128256 (the benchmark workload); the
     oracle checks a sample of 12 trees."""
     w = get_workload("eagle_v128k")
     inp = make_inputs(w, seed=3, device="cuda")
     trees = list(range(0, 128, 11))
+    check(tv, inp, trees=trees, unfused=unfused)
+
+
+@pytest.mark.parametrize("shape", ["4,8,3", "4,4,3", "4,2,2", "8,2,4", "8,1,3", "4,1,2"])
+def test_fused_launch_shapes(tv, shape, monkeypatch):
+    """Every launch shape of the fused kernel (consumer warps per CTA, CTAs per
+    tree, ring stages) gives the oracle's results (V=32000, EAGLE trees)."""
+    monkeypatch.setenv("TV_FUSED_PLAN", shape)
+    w = get_workload("eagle_v32k", batch=24)
+    inp = make_inputs(w, seed=24, device="cuda")
+    v = tv.Verifier(w.vocab, w.nodes, 24, "bf16")
+    got = v.launch_shape(24, w.nodes)
+    v.close()
+    ncw, c, st = (int(x) for x in shape.split(","))
+    assert got == (1, c, ncw, st)
+    check(tv, inp)
+
+
+@pytest.mark.parametrize("batch", [8, 40, 400])
+def test_default_launch_shapes(tv, batch):
+    """Batch sizes that select different default shapes (clusters of 8, 8 and
+    1 CTA, 4 or 8 consumer warps)."""
+    w = get_workload("eagle_v32k", batch=batch)
+    inp = make_inputs(w, seed=batch, device="cuda")
+    trees = list(range(0, batch, max(1, batch // 40)))
     check(tv, inp, trees=trees)
 
 
