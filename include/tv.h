@@ -204,6 +204,35 @@ int tv_last_phase_ms(tv_handle* h, float* ms);
 int tv_launch_shape(tv_handle* h, int B, int N, int* path, int* cluster, int* warps,
                     int* stages);
 
+/*
+ * tv_verify_batch_noalloc -- the same verification for callers that cannot
+ * allocate device memory (inside a CUDA-graph capture they do not own, under
+ * a memory pool that forbids new allocations, or where another allocator owns
+ * the device).  The paper has no counterpart: this is a deployment entry point.
+ *
+ * Needs no handle and allocates nothing: its scratch (internal-row list, row
+ * statistics, status word) is one fixed array of static device memory in the
+ * library image (about 0.8 MB, held by every GPU that loads the library until
+ * the process exits), used through the three-kernel path.  Limit:
+ * B * (N + 1) <= 65536 rows; larger calls return TV_ERR_CAPACITY and launch
+ * nothing.  The first call on a device makes that device current and looks up
+ * the array's device address (cudaGetSymbolAddress) once; issue that first
+ * call before any stream capture.  All calls share the array: each clears
+ * what must start at zero, but calls whose work overlaps on the GPU race on it
+ * and must not be issued.
+ *   device      : CUDA device ordinal (0..63) the pointers belong to.
+ *   vocab, logit_dtype : as in tv_create.
+ *   the rest    : as in tv_verify_batch (device pointers, caller-owned).
+ * Errors: TV_ERR_INVALID_ARG, TV_ERR_TEMPERATURE, TV_ERR_VOCAB,
+ * TV_ERR_CAPACITY, TV_ERR_DEVICE, TV_ERR_CUDA.
+ */
+int tv_verify_batch_noalloc(int device, int B, int N, int vocab, tv_dtype logit_dtype,
+                            const int32_t* parents, const int32_t* draft_tokens,
+                            const void* target_logits, const float* draft_probs,
+                            float temperature, const float* uniforms,
+                            int32_t* out_accepted_path, int32_t* out_accept_len,
+                            int32_t* out_bonus_token, void* cuda_stream);
+
 /* tv_destroy -- free the handle's workspace (synchronises its device). */
 int tv_destroy(tv_handle* h);
 

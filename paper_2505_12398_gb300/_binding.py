@@ -48,6 +48,8 @@ _SIGS = {
     "tv_last_phase_ms": (_I, [_P, ctypes.POINTER(ctypes.c_float)]),
     "tv_launch_shape": (_I, [_P, _I, _I, ctypes.POINTER(_I), ctypes.POINTER(_I),
                              ctypes.POINTER(_I), ctypes.POINTER(_I)]),
+    "tv_verify_batch_noalloc": (_I, [_I, _I, _I, _I, _I, _P, _P, _P, _P, _F, _P, _P, _P, _P,
+                                     _P]),
     "tv_strerror": (ctypes.c_char_p, [_I]),
     "tv_version": (_I, []),
 }
