@@ -40,6 +40,8 @@ def parse_args():
     ap.add_argument("--batch", type=int, default=None)
     ap.add_argument("--sigma", type=float, default=None)
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--path", choices=["auto", "persistent", "cluster", "three"], default="auto",
+                    help="kernel path of the handle (auto: the library's choice)")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -206,7 +208,7 @@ def main():
     B, R = inp.parents.shape
     N, V = R - 1, w.vocab
     lb = 2 if inp.logits.dtype == torch.bfloat16 else 4
-    v = tv.Verifier(V, N, B, "bf16" if lb == 2 else "fp32", device=dev.index)
+    v = tv.Verifier(V, N, B, "bf16" if lb == 2 else "fp32", device=dev.index, path=args.path)
     stream = torch.cuda.current_stream(dev)
 
     # decisions are a deterministic function of the inputs: one instrumented
@@ -215,7 +217,7 @@ def main():
                                      inp.temperature, inp.uniforms, debug=True)
     torch.cuda.synchronize(dev)
     row_bytes, trav_bytes = algorithmic_bytes(inp.parents, stats, V, lb)
-    fused, cluster, warps, stages = v.launch_shape(B, N)
+    path_code, cluster, warps, stages = v.launch_shape(B, N)
     a_bytes = row_bytes + trav_bytes
     mean_tau1 = float(tau_d.float().mean()) + 1.0
     passes_per_tree = float(stats[:, 1].float().mean())
@@ -303,8 +305,17 @@ def main():
 
     peak, peak_kind = measured_peaks()
     ph = [sum(p[i] for p in phase) / len(phase) for i in range(3)]
-    names = ["tv_prep_kernel", "tv_row_stats_kernel", "tv_traverse_kernel"]
-    kbytes = [0, row_bytes, trav_bytes]
+    if path_code == 0:
+        names = ["tv_prep_kernel", "tv_row_stats_kernel", "tv_traverse_kernel"]
+        kbytes = [0, row_bytes, trav_bytes]
+        launches_per_step = 3
+    else:
+        # one kernel reads every row the traversal needs; the first two
+        # phases are empty (their events are recorded back to back)
+        single = "tv_tree_kernel" if path_code == 1 else "tv_flow_kernel"
+        names = ["-", "-", single]
+        kbytes = [0, 0, a_bytes]
+        launches_per_step = 1
     dom = max(range(3), key=lambda i: ph[i])
     ms_step = total_ms_max / args.steps
     trees_s = B * world * args.steps / (total_ms_max / 1e3)
@@ -331,14 +342,15 @@ def main():
                    "temperature": w.temperature, "sigma": w.sigma, "seed": args.seed,
                    "l2": "flushed by a 256 MiB write before every timed step (untimed)",
                    "parallelism": f"dp{world} (independent trees per GPU)",
-                   "kernel_path": "fused" if fused else "three-kernel",
+                   "kernel_path": ["three-kernel", "cluster-per-tree",
+                                   "persistent"][path_code],
                    "ctas_per_tree": cluster, "consumer_warps": warps, "ring_stages": stages},
         "verified_logit_gbps": round(step_gbs, 2),
         "hbm_frac_step": round(step_gbs / peak, 4),
         "algorithmic_bytes_per_step": a_bytes,
         "mean_accept_len_tau_plus_1": round(mean_tau1, 4),
         "rejection_passes_per_tree": round(passes_per_tree, 3),
-        "phase_ms": {names[i]: round(ph[i], 6) for i in range(3)},
+        "phase_ms": {names[i]: round(ph[i], 6) for i in range(3) if names[i] != "-"},
         "roofline": {"bound": "hbm", "kernel": names[dom], "achieved": round(dom_gbs, 2),
                      "peak": peak, "unit": "GB/s", "frac": round(dom_gbs / peak, 4),
                      "peak_kind": peak_kind, "bytes_per_launch": kbytes[dom],
@@ -346,7 +358,7 @@ def main():
         "roofline_step": {"bound": "hbm", "achieved": round(step_gbs, 2), "peak": peak,
                           "unit": "GB/s", "frac": round(step_gbs / peak, 4)},
         "e2e": e2e,
-        "gpu_launches": 3 * args.steps,
+        "gpu_launches": launches_per_step * args.steps,
         "clocks": clocks,
         "cpu_baseline": cpu,
         "wall_s_timed_region": round(wall, 3),

@@ -69,15 +69,23 @@ enum {
   TV_STATUS_BAD_ROW = 64u      /* a target row the traversal needed has no finite logit */
 };
 
-/* Flags for tv_create. */
+/* Flags for tv_create.  At most one may be given; with none the library picks
+   the path (the persistent kernel when V % 8 == 0, else the three-kernel
+   path).  All paths compute the same results; the two single-kernel paths read
+   rows with bulk copies and need V % 8 == 0, other vocabularies always take
+   the three-kernel path. */
 enum {
   TV_FLAG_NONE = 0u,
-  /* Use the three-kernel path (row normalisers of every internal row, then one
-     CTA per tree) even when the fused single-kernel path is available.  The
-     fused path (one thread-block cluster per tree, rows read lazily through
-     bulk copies) needs V % 8 == 0; other vocabularies always take the
-     three-kernel path.  Both compute the same results. */
-  TV_FLAG_UNFUSED = 1u
+  /* Three kernels: row normalisers of every internal row, then one CTA per
+     tree. */
+  TV_FLAG_UNFUSED = 1u,
+  /* One kernel, one thread-block cluster per tree (rows read lazily, the
+     vocabulary split across the cluster's CTAs). */
+  TV_FLAG_CLUSTER = 2u,
+  /* One persistent cooperative kernel: each tree's serial control runs in an
+     owner CTA, and the vocabulary work of every step is cut into slices that
+     any CTA of the grid may process (load balancing across trees). */
+  TV_FLAG_PERSISTENT = 4u
 };
 
 /*
@@ -89,7 +97,8 @@ enum {
  *                may pass; 0 <= max_nodes <= 1023.
  *   max_batch  : largest B later calls may pass; >= 1.
  *   logit_dtype: element type of target_logits in later calls.
- *   flags      : TV_FLAG_NONE or TV_FLAG_UNFUSED.
+ *   flags      : TV_FLAG_NONE or one of TV_FLAG_UNFUSED, TV_FLAG_CLUSTER,
+ *                TV_FLAG_PERSISTENT.
  * Errors: TV_ERR_INVALID_ARG, TV_ERR_VOCAB, TV_ERR_CUDA, TV_ERR_DEVICE.
  */
 int tv_create(tv_handle** out, int device, int vocab, int max_nodes, int max_batch,
@@ -196,9 +205,10 @@ int tv_last_phase_ms(tv_handle* h, float* ms);
 
 /*
  * tv_launch_shape -- how a call with these B and N would run on this handle:
- * *path = 1 for the fused single-kernel path, 0 for the three-kernel path;
- * for the fused path also the thread-block cluster size (CTAs per tree), the
- * consumer warps per CTA and the ring stages.  Any output pointer may be NULL.
+ * *path = 0 for the three-kernel path, 1 for the cluster-per-tree kernel, 2
+ * for the persistent kernel; *cluster = CTAs per tree (cluster path; 1
+ * otherwise), *warps = consumer warps per CTA, *stages = ring stages (0 for
+ * the three-kernel path).  Any output pointer may be NULL.
  * Errors: TV_ERR_INVALID_ARG, TV_ERR_CAPACITY.
  */
 int tv_launch_shape(tv_handle* h, int B, int N, int* path, int* cluster, int* warps,

@@ -9,8 +9,8 @@ CPU path, and using the binding without the compiled library raises.
     path, tau, bonus = v.verify(parents, tokens, logits, draft_probs, 1.0, uniforms)
 """
 
-from ._binding import (TV_BF16, TV_FP32, TV_STATUS, LibraryError, Verifier,
+from ._binding import (PATH_FLAGS, TV_BF16, TV_FP32, TV_STATUS, LibraryError, Verifier,
                        library, library_path, status_names)
 
-__all__ = ["Verifier", "library", "library_path", "LibraryError", "TV_BF16", "TV_FP32",
-           "TV_STATUS", "status_names"]
+__all__ = ["Verifier", "library", "library_path", "LibraryError", "PATH_FLAGS", "TV_BF16",
+           "TV_FP32", "TV_STATUS", "status_names"]

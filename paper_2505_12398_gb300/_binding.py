@@ -7,6 +7,8 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 
 TV_BF16 = 0
 TV_FP32 = 1
+# tv_create flags: which kernel path a handle uses ("auto" lets the library pick)
+PATH_FLAGS = {"auto": 0, "three": 1, "cluster": 2, "persistent": 4}
 TV_STATUS = {
     "BAD_TREE": 1,
     "BAD_TOKEN": 2,
@@ -95,7 +97,7 @@ class Verifier:
     the handle's device with the dtypes and layouts of include/tv.h.
     """
 
-    def __init__(self, vocab, max_nodes, max_batch, logit_dtype="bf16", device=0, unfused=False):
+    def __init__(self, vocab, max_nodes, max_batch, logit_dtype="bf16", device=0, path="auto"):
         import torch
         self.lib = library()
         if logit_dtype in ("bf16", torch.bfloat16, TV_BF16):
@@ -107,8 +109,10 @@ class Verifier:
         self.vocab, self.max_nodes, self.max_batch = vocab, max_nodes, max_batch
         self.device = torch.device("cuda", device) if isinstance(device, int) else torch.device(device)
         h = ctypes.c_void_p()
+        if path not in PATH_FLAGS:
+            raise ValueError(f"unknown path {path!r}; one of {sorted(PATH_FLAGS)}")
         rc = self.lib.tv_create(ctypes.byref(h), self.device.index or 0, vocab, max_nodes,
-                                max_batch, self.dtype_code, 1 if unfused else 0)
+                                max_batch, self.dtype_code, PATH_FLAGS[path])
         if rc != 0:
             raise LibraryError("tv_create", rc, self.lib)
         self.handle = h
@@ -203,7 +207,8 @@ class Verifier:
         return [float(x) for x in ms]
 
     def launch_shape(self, B, N):
-        """(fused path?, CTAs per tree, consumer warps per CTA, ring stages)."""
+        """(path code, CTAs per tree, consumer warps per CTA, ring stages);
+        path code 0 = three kernels, 1 = cluster per tree, 2 = persistent."""
         out = [ctypes.c_int() for _ in range(4)]
         rc = self.lib.tv_launch_shape(self.handle, B, N, *[ctypes.byref(o) for o in out])
         if rc != 0:

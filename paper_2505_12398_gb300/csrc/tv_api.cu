@@ -24,11 +24,15 @@ struct tv_handle {
   int smem_per_sm = 0;
   int smem_per_block = 0;
   int force_ncw = 0, force_c = 0, force_stages = 0;   // tuning override (TV_FUSED_PLAN)
+  int flow_force[4] = {0, 0, 0, 0};                    // tuning override (TV_FLOW_PLAN)
   // device workspace
   int32_t* row_list = nullptr;   // [max_batch * (max_nodes + 1)]
   int32_t* n_rows = nullptr;     // [1]
   float2* stats = nullptr;       // [max_batch * (max_nodes + 1)]
   uint32_t* status = nullptr;    // [1]
+  void* flow_ws = nullptr;       // persistent kernel's queue and partials
+  size_t flow_ws_bytes = 0;
+  unsigned long long epoch = 0;  // per-call tag of the persistent kernel's queue
   // staging for tv_verify_batch_host (allocated on first use)
   char* stage = nullptr;
   size_t stage_bytes = 0;
@@ -42,6 +46,31 @@ namespace {
 
 constexpr int kMaxRows = 1024;   // N + 1
 constexpr int kMaxVocab = 1 << 28;
+constexpr unsigned kPathFlags = TV_FLAG_UNFUSED | TV_FLAG_CLUSTER | TV_FLAG_PERSISTENT;
+
+enum Path { kPathThree = 0, kPathCluster = 1, kPathPersistent = 2 };
+
+FlowPlan flow_plan(const tv_handle* h, int R) {
+  return tv_flow_plan(R, h->smem_per_sm, h->smem_per_block, h->flow_force[0], h->flow_force[1],
+                      h->flow_force[2], h->flow_force[3]);
+}
+
+// Smallest slice the persistent kernel may use on this handle (sizes its queue).
+int flow_min_slice(const tv_handle* h) {
+  const FlowPlan p = flow_plan(h, h->max_nodes + 1);
+  return p.slice_pass < p.slice_stats ? p.slice_pass : p.slice_stats;
+}
+
+Path choose_path(const tv_handle* h, int B, int R, FusedPlan* plan) {
+  if ((h->vocab % 8) != 0 || (h->flags & TV_FLAG_UNFUSED)) return kPathThree;
+  if (h->flags & TV_FLAG_CLUSTER) {
+    *plan = tv_fused_plan(B, R, h->vocab, h->sm_count, h->smem_per_sm, h->smem_per_block,
+                          h->force_ncw, h->force_c, h->force_stages);
+    return plan->ok ? kPathCluster : kPathThree;
+  }
+  if (!h->flow_ws || !flow_plan(h, R).ok) return kPathThree;
+  return kPathPersistent;
+}
 
 class DeviceGuard {
  public:
@@ -114,17 +143,22 @@ int verify_impl(tv_handle* h, int B, int N, const int32_t* parents, const int32_
   int grid = h->sm_count * 4;
   if (grid > rows) grid = rows;
   if (grid < 1) grid = 1;
-  const bool fused = (h->vocab % 8) == 0 && !(h->flags & TV_FLAG_UNFUSED);
   FusedPlan plan;
-  if (fused)
-    plan = tv_fused_plan(B, N + 1, h->vocab, h->sm_count, h->smem_per_sm, h->smem_per_block,
-                         h->force_ncw, h->force_c, h->force_stages);
-  if (fused && plan.ok) {
-    rc = tv_launch_fused(a, h->dtype == TV_BF16 ? 1 : 0, plan, static_cast<cudaStream_t>(stream),
-                         h->timing ? h->ev : nullptr);
+  const Path path = choose_path(h, B, N + 1, &plan);
+  const int bf16 = h->dtype == TV_BF16 ? 1 : 0;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  cudaEvent_t* ev = h->timing ? h->ev : nullptr;
+  if (path == kPathCluster) {
+    rc = tv_launch_fused(a, bf16, plan, st, ev);
+  } else if (path == kPathPersistent) {
+    FlowArgs f;
+    const FlowPlan fp = flow_plan(h, N + 1);
+    if (tv_flow_bind(h->flow_ws, h->flow_ws_bytes, B, N + 1, h->vocab, fp, &f) != 0)
+      return TV_ERR_CAPACITY;
+    f.epoch = ++h->epoch;
+    rc = tv_launch_flow(a, f, bf16, fp, h->sm_count, st, ev);
   } else {
-    rc = tv_launch_all(a, h->dtype == TV_BF16 ? 1 : 0, h->row_list, h->n_rows, grid,
-                       static_cast<cudaStream_t>(stream), h->timing ? h->ev : nullptr);
+    rc = tv_launch_all(a, bf16, h->row_list, h->n_rows, grid, st, ev);
   }
   if (rc == TV_OK && h->timing) h->timed_call = true;
   return rc;
@@ -141,7 +175,7 @@ int tv_create(tv_handle** out, int device, int vocab, int max_nodes, int max_bat
   if (vocab < 1 || vocab > kMaxVocab) return TV_ERR_VOCAB;
   if (max_nodes < 0 || max_nodes + 1 > kMaxRows || max_batch < 1) return TV_ERR_INVALID_ARG;
   if (logit_dtype != TV_BF16 && logit_dtype != TV_FP32) return TV_ERR_INVALID_ARG;
-  if (flags & ~TV_FLAG_UNFUSED) return TV_ERR_INVALID_ARG;
+  if ((flags & ~kPathFlags) || __builtin_popcount(flags) > 1) return TV_ERR_INVALID_ARG;
   int ndev = 0;
   if (cudaGetDeviceCount(&ndev) != cudaSuccess || device < 0 || device >= ndev) {
     cudaGetLastError();
@@ -168,6 +202,11 @@ int tv_create(tv_handle** out, int device, int vocab, int max_nodes, int max_bat
   // shape (tuning only; invalid values are ignored)
   if (const char* env = std::getenv("TV_FUSED_PLAN"))
     std::sscanf(env, "%d,%d,%d", &h->force_ncw, &h->force_c, &h->force_stages);
+  // TV_FLOW_PLAN="ncw,stages,slice_pass,slice_stats" does the same for the
+  // persistent kernel
+  if (const char* env = std::getenv("TV_FLOW_PLAN"))
+    std::sscanf(env, "%d,%d,%d,%d", &h->flow_force[0], &h->flow_force[1], &h->flow_force[2],
+                &h->flow_force[3]);
   DeviceGuard guard(device);
   if (!guard.ok()) {
     delete h;
@@ -179,6 +218,13 @@ int tv_create(tv_handle** out, int device, int vocab, int max_nodes, int max_bat
             cudaMalloc(&h->stats, rows * sizeof(float2)) == cudaSuccess &&
             cudaMalloc(&h->status, sizeof(uint32_t)) == cudaSuccess &&
             cudaMemset(h->status, 0, sizeof(uint32_t)) == cudaSuccess;
+  if (ok && (vocab % 8) == 0 && !(flags & (TV_FLAG_UNFUSED | TV_FLAG_CLUSTER))) {
+    // the queue's publication tags start at zero; calls use epochs 1, 2, ...
+    h->flow_ws_bytes = tv_flow_workspace_bytes(max_batch, max_nodes + 1, vocab,
+                                               flow_min_slice(h));
+    ok = cudaMalloc(&h->flow_ws, h->flow_ws_bytes) == cudaSuccess &&
+         cudaMemset(h->flow_ws, 0, h->flow_ws_bytes) == cudaSuccess;
+  }
   if (!ok) {
     cudaGetLastError();
     tv_destroy(h);
@@ -331,16 +377,14 @@ int tv_launch_shape(tv_handle* h, int B, int N, int* path, int* cluster, int* wa
                     int* stages) {
   if (!h || B < 0 || N < 0) return TV_ERR_INVALID_ARG;
   if (B > h->max_batch || N > h->max_nodes) return TV_ERR_CAPACITY;
-  const bool fused = (h->vocab % 8) == 0 && !(h->flags & TV_FLAG_UNFUSED);
   FusedPlan plan;
-  if (fused)
-    plan = tv_fused_plan(B, N + 1, h->vocab, h->sm_count, h->smem_per_sm, h->smem_per_block,
-                         h->force_ncw, h->force_c, h->force_stages);
-  const bool f = fused && plan.ok;
-  if (path) *path = f ? 1 : 0;
-  if (cluster) *cluster = f ? plan.C : 1;
-  if (warps) *warps = f ? plan.ncw : 16;
-  if (stages) *stages = f ? plan.stages : 0;
+  const Path p = choose_path(h, B, N + 1, &plan);
+  if (path) *path = (int)p;
+  if (cluster) *cluster = (p == kPathCluster) ? plan.C : 1;
+  const FlowPlan fp = flow_plan(h, N + 1);
+  if (warps) *warps = (p == kPathCluster) ? plan.ncw : (p == kPathPersistent ? fp.ncw : 16);
+  if (stages)
+    *stages = (p == kPathCluster) ? plan.stages : (p == kPathPersistent ? fp.stages : 0);
   return TV_OK;
 }
 
@@ -355,6 +399,7 @@ int tv_destroy(tv_handle* h) {
     cudaFree(h->n_rows);
     cudaFree(h->stats);
     cudaFree(h->status);
+    if (h->flow_ws) cudaFree(h->flow_ws);
     if (h->stage) cudaFree(h->stage);
     cudaGetLastError();
   }

@@ -49,3 +49,55 @@ size_t tv_traverse_smem_bytes(int R, int V);
 // between the kernels and after the last one.
 int tv_launch_all(const TravArgs& a, int logit_is_bf16, int* row_list, int* n_rows,
                   int stats_grid, cudaStream_t stream, cudaEvent_t* events);
+
+// ---- persistent load-balanced kernel (tv_flow.cu) ----
+
+// One slot of the persistent kernel's work queue: a slice of one tree's
+// current vocabulary job, self-contained so that a claim is one 48-byte read.
+struct __align__(64) FlowItem {
+  int tree, node, row, slice;   // tree, target row, row index within the job, slice
+  int kind, slice_len, nmask, pad0;
+  float alpha1, beta, rowmax, pad1;
+  unsigned long long tag;       // epoch << 32 | slot, stored after the rest
+  unsigned long long pad2;
+};
+
+// Device workspace of the persistent kernel (carved by tv_flow_bind).
+struct FlowArgs {
+  unsigned* ctr;                 // queue tail, head, trees done, next tree, abort, CTAs out
+                                 // (zero between calls: the last CTA out resets them)
+  FlowItem* items;               // [cap] queue slots
+  int* job_mtok;                 // [B][R] removed tokens of a tree's current job row
+  float* job_mval;               // [B][R] their stored masses (bonus residual)
+  unsigned long long* part;      // [B][R][Kmax] partial (x, y) per (row, slice); all ones
+                                 // until the slice is done
+  unsigned* finished;            // [B] epoch of the call that finished the tree
+  float2* tiles;                 // [B][ntiles] per-tile sums of the bonus draw
+  unsigned long long epoch;      // differs between calls sharing the workspace
+  int cap, R, Kmax, ntiles;
+  int slice_pass, slice_stats;   // tokens per slice (multiples of 256)
+};
+
+// Launch shape of the persistent kernel.
+struct FlowPlan {
+  int ncw = 4;                   // consumer warps per CTA (4 or 8)
+  int stages = 3;                // ring stages of 3 KB per consumer warp
+  int slice_pass = 8192;         // tokens per slice of a pass / bonus draw
+  int slice_stats = 16384;       // tokens per slice of a row normaliser
+  size_t smem = 0;
+  bool ok = false;
+};
+
+// Default plan for R = N+1 rows (tuning overrides: force_* > 0).
+FlowPlan tv_flow_plan(int R, int smem_per_sm, int smem_per_block, int force_ncw,
+                      int force_stages, int force_slice_pass, int force_slice_stats);
+// Workspace for slices of at least `min_slice` tokens.
+size_t tv_flow_workspace_bytes(int B, int R, int V, int min_slice);
+// Carves the workspace; 0 on success, TV_ERR_CAPACITY if `bytes` is too small.
+int tv_flow_bind(void* base, size_t bytes, int B, int R, int V, const FlowPlan& plan,
+                 FlowArgs* f);
+// Queues the cooperative persistent kernel.  The workspace must have been
+// zeroed once before the first call.  Requires V % 8 == 0.  `events` as for
+// tv_launch_fused.
+int tv_launch_flow(const TravArgs& a, FlowArgs f, int logit_is_bf16, const FlowPlan& plan,
+                   int sm_count, cudaStream_t stream, cudaEvent_t* events);

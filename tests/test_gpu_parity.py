@@ -21,11 +21,14 @@ def tv():
     return tv
 
 
-def run_gpu(tv, inp, debug=True, unfused=False):
+PATHS = ["persistent", "cluster", "three"]
+
+
+def run_gpu(tv, inp, debug=True, path="auto"):
     B, R = inp.parents.shape
     V = inp.logits.shape[-1]
     dt = "bf16" if inp.logits.dtype == torch.bfloat16 else "fp32"
-    v = tv.Verifier(V, R - 1, B, dt, unfused=unfused)
+    v = tv.Verifier(V, R - 1, B, dt, path=path)
     out = v.verify(inp.parents, inp.tokens, inp.logits, inp.draft_probs, inp.temperature,
                    inp.uniforms, debug=debug)
     torch.cuda.synchronize()
@@ -34,8 +37,8 @@ def run_gpu(tv, inp, debug=True, unfused=False):
     return [o.cpu().numpy() for o in out], status
 
 
-def check(tv, inp, trees=None, max_tie_frac=0.25, unfused=False):
-    (path, tau, bonus, node_p, stats), status = run_gpu(tv, inp, unfused=unfused)
+def check(tv, inp, trees=None, max_tie_frac=0.25, path="auto"):
+    (path, tau, bonus, node_p, stats), status = run_gpu(tv, inp, path=path)
     if trees is None:
         trees = list(range(inp.parents.shape[0]))
     par, tok, lg, dp, un = to_numpy_inputs(inp, trees)
@@ -50,39 +53,40 @@ def check(tv, inp, trees=None, max_tie_frac=0.25, unfused=False):
     return summ, status
 
 
-@pytest.mark.parametrize("unfused", [False, True])
-def test_tiny_many_seeds(tv, unfused):
+@pytest.mark.parametrize("path", PATHS)
+def test_tiny_many_seeds(tv, path):
     """The 7-node, V=64, fp32 tree, 512 draws of logits / tree / uniforms."""
     w = get_workload("tiny", batch=512)
     inp = make_inputs(w, seed=0, device="cuda")
-    summ, status = check(tv, inp, unfused=unfused)
+    summ, status = check(tv, inp, path=path)
     assert summ["exact"] >= 0.9 * summ["trees"]
     assert status & ~16 == 0
 
 
 @pytest.mark.parametrize("name", ["chain8", "binary4"])
 @pytest.mark.parametrize("sigma", [0.5, 1.0, 2.0])
-def test_chain_and_binary(tv, name, sigma):
+@pytest.mark.parametrize("path", ["persistent", "cluster"])
+def test_chain_and_binary(tv, name, sigma, path):
     w = get_workload(name, sigma=sigma)
     inp = make_inputs(w, seed=1, device="cuda")
-    check(tv, inp)
+    check(tv, inp, path=path)
 
 
-@pytest.mark.parametrize("unfused", [False, True])
-def test_eagle_v32k_all_trees(tv, unfused):
+@pytest.mark.parametrize("path", PATHS)
+def test_eagle_v32k_all_trees(tv, path):
     w = get_workload("eagle_v32k")
     inp = make_inputs(w, seed=2, device="cuda")
-    check(tv, inp, unfused=unfused)
+    check(tv, inp, path=path)
 
 
-@pytest.mark.parametrize("unfused", [False, True])
-def test_eagle_v128k_sampled(tv, unfused):
+@pytest.mark.parametrize("path", PATHS)
+def test_eagle_v128k_sampled(tv, path):
     """Full batch of 128 trees at V=128256 (the benchmark workload); the
     oracle checks a sample of 12 trees."""
     w = get_workload("eagle_v128k")
     inp = make_inputs(w, seed=3, device="cuda")
     trees = list(range(0, 128, 11))
-    check(tv, inp, trees=trees, unfused=unfused)
+    check(tv, inp, trees=trees, path=path)
 
 
 @pytest.mark.parametrize("shape", ["4,8,3", "4,4,3", "4,2,2", "8,2,4", "8,1,3", "4,1,2"])
@@ -92,34 +96,37 @@ def test_fused_launch_shapes(tv, shape, monkeypatch):
     monkeypatch.setenv("TV_FUSED_PLAN", shape)
     w = get_workload("eagle_v32k", batch=24)
     inp = make_inputs(w, seed=24, device="cuda")
-    v = tv.Verifier(w.vocab, w.nodes, 24, "bf16")
+    v = tv.Verifier(w.vocab, w.nodes, 24, "bf16", path="cluster")
     got = v.launch_shape(24, w.nodes)
     v.close()
     ncw, c, st = (int(x) for x in shape.split(","))
     assert got == (1, c, ncw, st)
-    check(tv, inp)
+    check(tv, inp, path="cluster")
 
 
-@pytest.mark.parametrize("batch", [8, 40, 400])
-def test_default_launch_shapes(tv, batch):
-    """Batch sizes that select different default shapes (clusters of 8, 8 and
-    1 CTA, 4 or 8 consumer warps)."""
+@pytest.mark.parametrize("batch", [1, 8, 40, 400, 1000])
+@pytest.mark.parametrize("path", ["persistent", "cluster"])
+def test_default_launch_shapes(tv, batch, path):
+    """Batch sizes that select different default cluster shapes (clusters of
+    8, 8 and 1 CTA, 4 or 8 consumer warps) and, for the persistent kernel,
+    fewer and more trees than CTAs."""
     w = get_workload("eagle_v32k", batch=batch)
     inp = make_inputs(w, seed=batch, device="cuda")
     trees = list(range(0, batch, max(1, batch // 40)))
-    check(tv, inp, trees=trees)
+    check(tv, inp, trees=trees, path=path)
 
 
-@pytest.mark.parametrize("V", [1000, 1003, 257, 8])
+@pytest.mark.parametrize("V", [1000, 1003, 257, 8, 8200, 16392])
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
-def test_ragged_vocab(tv, V, dtype):
+@pytest.mark.parametrize("path", ["auto", "cluster"])
+def test_ragged_vocab(tv, V, dtype, path):
     """Vocabularies that are not a multiple of the 8-element chunk or of the
     256-element bonus tile exercise the scalar-load path and the tails."""
     from workloads.synth import Workload
     w = Workload("ragged", 48, V, levels=(2, 3, 2), branching=(2, 2, 1),
                  logit_dtype=dtype, sigma=1.0)
     inp = make_inputs(w, seed=V, device="cuda")
-    check(tv, inp)
+    check(tv, inp, path=path)
 
 
 def test_root_only_trees(tv):
@@ -143,7 +150,8 @@ def test_temperatures(tv, T):
     check(tv, inp)
 
 
-def test_invalid_trees_flagged(tv):
+@pytest.mark.parametrize("path", PATHS)
+def test_invalid_trees_flagged(tv, path):
     from workloads.synth import Workload
     w = Workload("inv", 6, 512, levels=(2, 2), branching=(2, 1), logit_dtype=torch.float32)
     inp = make_inputs(w, seed=9, device="cuda")
@@ -153,9 +161,9 @@ def test_invalid_trees_flagged(tv):
     inp.parents[4, 0] = 0            # root with a parent
     par = inp.parents[5].tolist()
     inp.draft_probs[5, par[1], inp.tokens[5, 1]] = 0.0   # zero draft probability
-    (path, tau, bonus, node_p, stats), status = run_gpu(tv, inp)
+    (acc_path, tau, bonus, node_p, stats), status = run_gpu(tv, inp, path=path)
     assert tau[0] >= 0
-    assert (tau[1:] == -1).all() and (bonus[1:] == -1).all() and (path[1:] == -1).all()
+    assert (tau[1:] == -1).all() and (bonus[1:] == -1).all() and (acc_path[1:] == -1).all()
     assert status & 1 and status & 2 and status & 4 and status & 8
     p2, t2, l2, d2, u2 = to_numpy_inputs(inp)
     _, otau, _, _ = verify_batch(p2, t2, l2, d2, inp.temperature, u2)

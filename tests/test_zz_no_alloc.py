@@ -50,7 +50,7 @@ def noalloc(tv, inp, dtype_code, stream=None):
 
 def reference(tv, inp, dtype):
     B, R = inp.parents.shape
-    v = tv.Verifier(inp.logits.shape[-1], R - 1, B, dtype, unfused=True)
+    v = tv.Verifier(inp.logits.shape[-1], R - 1, B, dtype, path="three")
     out = v.verify(inp.parents, inp.tokens, inp.logits, inp.draft_probs, inp.temperature,
                    inp.uniforms)
     torch.cuda.synchronize()
