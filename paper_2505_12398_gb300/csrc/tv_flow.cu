@@ -9,23 +9,31 @@
 // slices that are published to a global work queue and processed by whichever
 // CTA holds the slot's ticket.  The owner combines the slices' partial results
 // in a fixed order (results do not depend on which CTA did what) and advances
-// its tree.  The kernel's time is then set by the slowest tree's chain of
-// jobs, each taking a few microseconds, instead of by its total bytes.
+// its tree.
+//
+// Each CTA is warp-specialised:
+//   * an owner warp runs the serial control of the CTA's current tree (tree
+//     set-up, combining partials, Eqs. (1)-(3), posting the next job);
+//   * a producer warp takes tickets, reads the queued slices and streams them
+//     into a shared-memory ring with 1-D bulk copies (TMA), one slice ahead;
+//   * NCW consumer warps reduce the ring stages and write each slice's
+//     partial result.
+// So the serial control of one tree overlaps the streaming of others, and
+// consecutive slices of a CTA stream back to back.
 //
 // One cooperative launch keeps all CTAs resident, so CTAs may wait on work
 // published by others; every wait is bounded, and a global abort flag ends
-// the kernel cleanly if one ever gives up.  Inside a CTA, a producer warp
-// streams a slice into a shared-memory ring with 1-D bulk copies (TMA) and
-// four consumer warps reduce it.
+// the kernel cleanly if one ever gives up.  Consumer warps synchronise only
+// through mbarriers (bounded waits), never through bar.sync, so a warp that
+// gives up cannot leave the others blocked.
 //
 // Queue protocol: a poster reserves a range of slots with one atomicAdd on
 // the tail, writes the slots' bodies, fences, then stores each slot's tag
-// (call epoch, slot number).  A CTA takes a ticket -- the next slot number,
-// one atomicAdd on the head -- and processes that slot once its tag appears,
-// doing its own tree's work meanwhile.  Slots are never reused within a call
-// (the queue holds every item the call can post), so a ticket past the last
-// item just waits for the end of the call.  Polls are relaxed loads issued
-// together; a positive poll is followed by one acquire fence.
+// (call epoch, slot number).  A producer takes a ticket -- the next slot
+// number, one atomicAdd on the head -- and processes that slot once its tag
+// appears.  Slots are never reused within a call; when the last tree is done
+// its owner writes an exit tag into every slot a ticket may still point to.
+// A slice's partial is one 64-bit store that doubles as its completion flag.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -40,6 +48,7 @@ namespace flow {
 using namespace tvk::fused;
 
 constexpr int kMaxNCW = 8;
+constexpr int kSlots = 2;           // queued slices a CTA holds: one streaming, one ahead
 constexpr int kPBuf = 256;          // partials of a job kept in shared memory by the poll
 constexpr unsigned long long kNoPart = ~0ull;   // a partial slot not written yet
 constexpr unsigned kNoTicket = 0xffffffffu;
@@ -47,24 +56,30 @@ constexpr unsigned long long kExitTag = 0x80000000ull;   // tag bit: no more ite
 constexpr int kMaxGrid = 4096;      // tickets taken past the last item: one per CTA at most
 constexpr unsigned long long kIdleNs = 2000000000ull;   // 2 s without progress: abort
 
-enum : int { kActIdle = 0, kActItem = 1, kActCombine = 2, kActNewTree = 3, kActExit = 4 };
 enum : int {
   kCtrTail = 0, kCtrHead = 1, kCtrDone = 2, kCtrNextTree = 3, kCtrAbort = 4, kCtrExit = 5,
   kNumCtr = 6
 };
+enum : int { kStageFirst = 1, kStageLast = 2, kStageExit = 4 };
+
+// A queued slice as held by a CTA (the masks live in shared arrays of R).
+struct ItemSlot {
+  int b, node, row, slice;
+  int kind, slice_len, nmask, pad0;
+  float alpha1, beta, rowmax, pad1;
+};
+
+struct StageMeta {
+  int slot, x, n, flags;
+};
 
 struct Shared {
-  int act;
-  int my_tree;          // tree owned by this CTA (-1: none)
-  int outstanding;      // items of the own tree's current job (0: none)
-  unsigned ticket;      // queue slot this CTA processes next (kNoTicket: none)
-  int jkind, jrows, jK, jslice;   // own tree's current job, for the combine
-  int4 it[3];           // body of the item being processed
-  int trees_left;       // the next-tree counter may still be below B
-  Ctl ctl;              // serial control state of the own tree
-  float red_a[kMaxNCW], red_b[kMaxNCW];
-  float out_x, out_y;   // partial result of the item
-  float2 pbuf[kPBuf];   // the own job's partials, as read by the poll
+  ItemSlot slots[kSlots];
+  StageMeta meta[kMaxStages];
+  float2 red[kMaxStages][kMaxNCW];   // per-warp partials of the slice ending in a stage
+  Ctl ctl;                           // serial control state of the own tree (owner warp)
+  float2 pbuf[kPBuf];                // the own job's partials, as read by the poll
+  int jkind, jrows, jK, jslice, outstanding;
 };
 
 __device__ __forceinline__ unsigned ld_relaxed_u32(const unsigned* p) {
@@ -100,15 +115,414 @@ __device__ __forceinline__ unsigned long long global_ns() {
   return t;
 }
 
-// Ends the whole kernel cleanly: every CTA sees the flag at its next decision.
+// Ends the whole kernel cleanly: every role sees the flag at its next poll.
 __device__ __forceinline__ void raise_abort(const TravArgs& a, const FlowArgs& f) {
   atomicOr(a.status, 32u);
   atomicExch(&f.ctr[kCtrAbort], 1u);
 }
 
-// --------------------------------------------------------------- posting --
+// An mbarrier wait whose outcome is the same for every lane of the warp (a
+// lane that gave up makes the whole warp give up), so that no lane is left
+// alone at a later warp-wide operation.
+__device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity) {
+  return __all_sync(0xffffffffu, mbar_wait(bar, parity) ? 1 : 0) != 0;
+}
 
-// Publishes the own tree's current job (ctl.job) as slice items; warp 0.
+// Sleep of an idle poller: 32 ns doubling to 256 ns; false once the wait has
+// lasted kIdleNs (the caller aborts).
+struct Backoff {
+  unsigned nap = 32u;
+  unsigned long long since = 0ull;
+  __device__ __forceinline__ void reset() {
+    nap = 32u;
+    since = 0ull;
+  }
+  __device__ __forceinline__ bool idle() {
+    const unsigned long long now = global_ns();
+    if (since == 0ull) since = now;
+    else if (now - since > kIdleNs) return false;
+    __nanosleep(nap);
+    if (nap < 256u) nap <<= 1;
+    return true;
+  }
+};
+
+// ------------------------------------------------------------- shapes --
+
+template <typename L, int kNCW>
+struct Shape {
+  static constexpr int kConsumers = kNCW * 32;
+  static constexpr int kThreads = kConsumers + 64;   // + producer + owner warps
+  static constexpr int kStageBytes = stage_bytes(kNCW);
+  static constexpr int kSweep = kConsumers * kChunk;
+  static constexpr int kLB = L::kBytes;
+  // tokens per stage: target and draft values together, or target only
+  static constexpr int kPairElems = kStageBytes / (kLB + 4) / kTileElems * kTileElems;
+  static constexpr int kRowElems = kStageBytes / kLB;
+};
+
+struct Smem {
+  char* ring;
+  TreeSmem s;
+  int* mtok;     // [kSlots][R] removed tokens of the held slices
+  float* mval;   // [kSlots][R] their stored masses
+  uint64_t* full_bar;
+  uint64_t* empty_bar;
+  uint64_t* slot_free;
+  uint64_t* red_bar;
+  Shared* sh;
+};
+
+// ------------------------------------------------------------ producer --
+
+template <typename L, int kNCW>
+__device__ void producer_role(const TravArgs& a, const FlowArgs& f, const Smem& m,
+                              int n_stages, int lane) {
+  using S = Shape<L, kNCW>;
+  using E = typename L::elem;
+  const int R = a.N + 1, V = a.V, B = a.B;
+  const E* logits = reinterpret_cast<const E*>(a.logits);
+  int stage = 0, phase = 0, slot = 0, slot_phase = 0;
+  unsigned ticket = kNoTicket, polls = 0u;
+  Backoff wait;
+  bool aborted = false;
+  for (;;) {
+    // ---- wait for the ticket's slot to be published (lane 0) ----
+    int cmd = 0;   // 0: keep polling, 1: a slice, 2: stop
+    if (lane == 0) {
+      if (ticket == kNoTicket) {
+        if (ld_relaxed_u32(&f.ctr[kCtrDone]) >= (unsigned)B) cmd = 2;   // nothing will come
+        else ticket = atomicAdd(&f.ctr[kCtrHead], 1u);
+      }
+      if (cmd == 0) {
+        const unsigned long long want = (f.epoch << 32) | (unsigned long long)ticket;
+        const unsigned long long tag =
+            (ticket < (unsigned)f.cap) ? ld_relaxed_u64(&f.items[ticket].tag) : 0ull;
+        if ((++polls & 31u) == 0u && ld_relaxed_u32(&f.ctr[kCtrAbort])) {
+          cmd = 2;
+        } else if (tag == want) {
+          fence_gpu();
+          cmd = 1;
+          wait.reset();
+        } else if (tag == (want | kExitTag)) {
+          cmd = 2;
+        } else if (!wait.idle()) {
+          raise_abort(a, f);
+          cmd = 2;
+        }
+      }
+    }
+    cmd = __shfl_sync(0xffffffffu, cmd, 0);
+    if (cmd == 2) break;
+    if (cmd == 0) continue;
+
+    // ---- copy the slice's description into a free slot ----
+    int ok = 1;
+    if (lane == 0) ok = mbar_wait(&m.slot_free[slot], slot_phase ^ 1) ? 1 : 0;
+    ok = __shfl_sync(0xffffffffu, ok, 0);
+    if (!ok) {
+      if (lane == 0) raise_abort(a, f);
+      aborted = true;
+      break;
+    }
+    ItemSlot& it = m.sh->slots[slot];
+    int b = 0, nmask = 0;
+    if (lane == 0) {
+      const int4* bp = reinterpret_cast<const int4*>(f.items + ticket);
+      const int4 w0 = __ldcg(bp), w1 = __ldcg(bp + 1), w2 = __ldcg(bp + 2);
+      it.b = w0.x; it.node = w0.y; it.row = w0.z; it.slice = w0.w;
+      it.kind = w1.x; it.slice_len = w1.y; it.nmask = w1.z;
+      it.alpha1 = __int_as_float(w2.x); it.beta = __int_as_float(w2.y);
+      it.rowmax = __int_as_float(w2.z);
+      b = w0.x;
+      nmask = w1.z;
+      ticket = kNoTicket;
+    }
+    b = __shfl_sync(0xffffffffu, b, 0);
+    nmask = __shfl_sync(0xffffffffu, nmask, 0);
+    for (int q = lane; q < nmask; q += 32) {
+      m.mtok[slot * R + q] = __ldcg(f.job_mtok + (size_t)b * R + q);
+      m.mval[slot * R + q] = __ldcg(f.job_mval + (size_t)b * R + q);
+    }
+    __syncwarp();
+
+    // ---- stream it through the ring ----
+    if (lane == 0) {
+      const bool pair = (it.kind == kJobPass || it.kind == kJobBonusRes);
+      const int per = pair ? S::kPairElems : S::kRowElems;
+      const int x0 = it.slice * it.slice_len;
+      const int x1 = min(V, x0 + it.slice_len);
+      const size_t row = ((size_t)b * R + it.node) * (size_t)V;
+      for (int x = x0; x < x1; x += per) {
+        const int n = min(per, x1 - x);
+        if (!mbar_wait(&m.empty_bar[stage], phase ^ 1)) {
+          raise_abort(a, f);
+          aborted = true;
+          break;
+        }
+        m.sh->meta[stage] = StageMeta{slot, x, n, (x == x0 ? kStageFirst : 0) |
+                                                      (x + n >= x1 ? kStageLast : 0)};
+        char* dst = m.ring + (size_t)stage * S::kStageBytes;
+        const uint32_t lbytes = (uint32_t)n * S::kLB;
+        const uint32_t qbytes = pair ? (uint32_t)n * 4u : 0u;
+        mbar_arrive_expect_tx(&m.full_bar[stage], lbytes + qbytes);
+        tma_load_1d(dst, logits + row + x, lbytes, &m.full_bar[stage]);
+        if (pair)
+          tma_load_1d(dst + (size_t)S::kPairElems * S::kLB, a.draft_probs + row + x, qbytes,
+                      &m.full_bar[stage]);
+        if (++stage == n_stages) { stage = 0; phase ^= 1; }
+      }
+    }
+    stage = __shfl_sync(0xffffffffu, stage, 0);
+    phase = __shfl_sync(0xffffffffu, phase, 0);
+    if (__shfl_sync(0xffffffffu, aborted ? 1 : 0, 0)) break;
+    if (++slot == kSlots) { slot = 0; slot_phase ^= 1; }
+  }
+  // ---- tell the consumers to stop ----
+  if (lane == 0 && !aborted) {
+    if (mbar_wait(&m.empty_bar[stage], phase ^ 1)) {
+      m.sh->meta[stage] = StageMeta{0, 0, 0, kStageExit};
+      mbar_arrive(&m.full_bar[stage]);
+    } else {
+      raise_abort(a, f);
+    }
+  }
+  __syncwarp();
+}
+
+// ------------------------------------------------------------ consumers --
+
+template <typename L, int kNCW>
+__device__ void consumer_role(const TravArgs& a, const FlowArgs& f, const Smem& m,
+                              int n_stages, int wid, int lane) {
+  using S = Shape<L, kNCW>;
+  using E = typename L::elem;
+  const int R = a.N + 1, V = a.V;
+  const float c_hi = a.c_hi, c_lo = a.c_lo;
+  const float2 ch = make_float2(c_hi, c_hi), cl = make_float2(c_lo, c_lo);
+  int stage = 0, phase = 0;
+  unsigned red_phase = 0u;   // parity bit per stage of red_bar (warp 0 waits on it)
+  // the slice in progress
+  int kind = 0, b = 0, row_idx = 0, slice = 0, nmask = 0, slot = 0, x0 = 0, x1 = 0;
+  float alpha1 = 0.f, beta = 0.f, rowmax = 0.f;
+  float m_run = TV_NEG_INF;
+  Comp acc;
+  int mp = 0;
+  for (;;) {
+    if (!mbar_wait_warp(&m.full_bar[stage], phase)) {
+      if (lane == 0) raise_abort(a, f);
+      break;
+    }
+    const StageMeta meta = m.sh->meta[stage];
+    if (meta.flags & kStageExit) break;
+    if (meta.flags & kStageFirst) {
+      const ItemSlot& it = m.sh->slots[meta.slot];
+      kind = it.kind; b = it.b; row_idx = it.row; slice = it.slice; nmask = it.nmask;
+      alpha1 = it.alpha1; beta = it.beta; rowmax = it.rowmax;
+      slot = meta.slot;
+      x0 = slice * it.slice_len;
+      x1 = min(V, x0 + it.slice_len);
+      m_run = TV_NEG_INF;
+      acc = Comp();
+      mp = 0;
+    }
+    const int* mtok = m.mtok + slot * R;
+    const float* mval = m.mval + slot * R;
+    const int x = meta.x, n = meta.n;
+    const char* buf = m.ring + (size_t)stage * S::kStageBytes;
+    const E* lb = reinterpret_cast<const E*>(buf);
+    const float* qb = reinterpret_cast<const float*>(buf + (size_t)S::kPairElems * S::kLB);
+    for (int t0 = wid * kTileElems; t0 < n; t0 += S::kSweep) {
+      const int e0 = t0 + lane * kChunk;
+      const bool valid = e0 < n;
+      const int xg = x + e0;
+      float v[8];
+      float2 vp[4];
+      if constexpr (S::kLB == 2) {
+        if (valid) bf16x8_pairs(lds128(lb + e0), vp);
+        else {
+#pragma unroll
+          for (int k2 = 0; k2 < 4; ++k2) vp[k2] = make_float2(-9984.f, -9984.f);
+        }
+#pragma unroll
+        for (int k2 = 0; k2 < 4; ++k2) { v[2 * k2] = vp[k2].x; v[2 * k2 + 1] = vp[k2].y; }
+      } else {
+        if (valid) {
+          const uint4 a4 = lds128(lb + e0);
+          const uint4 b4 = lds128(lb + e0 + 4);
+          v[0] = __uint_as_float(a4.x); v[1] = __uint_as_float(a4.y);
+          v[2] = __uint_as_float(a4.z); v[3] = __uint_as_float(a4.w);
+          v[4] = __uint_as_float(b4.x); v[5] = __uint_as_float(b4.y);
+          v[6] = __uint_as_float(b4.z); v[7] = __uint_as_float(b4.w);
+        } else {
+#pragma unroll
+          for (int k2 = 0; k2 < 8; ++k2) v[k2] = TV_NEG_INF;
+        }
+      }
+      if (kind == kJobStats) {
+        if (valid) {
+          float cm = v[0];
+#pragma unroll
+          for (int k2 = 1; k2 < 8; ++k2) cm = fmaxf(cm, v[k2]);
+          if (cm > m_run) {
+            if (m_run != TV_NEG_INF) {
+              const float sc = L::exp_rel(m_run, cm, c_hi, c_lo);
+              acc.s *= sc;
+              acc.c *= sc;
+            }
+            m_run = cm;
+          }
+          float sum;
+          if constexpr (S::kLB == 2) {
+            const float2 mm = make_float2(-m_run, -m_run);
+            float2 e[4];
+#pragma unroll
+            for (int k2 = 0; k2 < 4; ++k2) e[k2] = exp2_split_x2(__fadd2_rn(vp[k2], mm), ch, cl);
+            const float2 s2 = __fadd2_rn(__fadd2_rn(e[0], e[1]), __fadd2_rn(e[2], e[3]));
+            sum = s2.x + s2.y;
+          } else {
+            float t[8];
+#pragma unroll
+            for (int k2 = 0; k2 < 8; ++k2) t[k2] = L::exp_rel(v[k2], m_run, c_hi, c_lo);
+            sum = sum8(t);
+          }
+          acc.add(sum);
+        }
+      } else if (kind == kJobBonusLeaf) {
+        float lm = v[0];
+#pragma unroll
+        for (int k2 = 1; k2 < 8; ++k2) lm = fmaxf(lm, v[k2]);
+        const float tm = warp_max(lm);
+        float t[8];
+#pragma unroll
+        for (int k2 = 0; k2 < 8; ++k2) t[k2] = L::exp_pass(v[k2], tm, c_hi, c_lo);
+        const float ts = warp_sum(valid ? sum8(t) : 0.f);
+        if (lane == 0)
+          __stcg(f.tiles + (size_t)b * f.ntiles + (x + t0) / kTileElems, make_float2(ts, tm));
+      } else {
+        float q[8];
+        if (valid) {
+          const uint4 qa = lds128(qb + e0);
+          const uint4 qc = lds128(qb + e0 + 4);
+          q[0] = __uint_as_float(qa.x); q[1] = __uint_as_float(qa.y);
+          q[2] = __uint_as_float(qa.z); q[3] = __uint_as_float(qa.w);
+          q[4] = __uint_as_float(qc.x); q[5] = __uint_as_float(qc.y);
+          q[6] = __uint_as_float(qc.z); q[7] = __uint_as_float(qc.w);
+        } else {
+#pragma unroll
+          for (int k2 = 0; k2 < 8; ++k2) q[k2] = 0.f;
+        }
+        float t[8];
+        if constexpr (S::kLB == 2) {
+          const float2 mm = make_float2(-rowmax, -rowmax);
+          const float2 al2 = make_float2(alpha1, alpha1);
+          const float2 nb2 = make_float2(-beta, -beta);
+#pragma unroll
+          for (int k2 = 0; k2 < 4; ++k2) {
+            const float2 e = exp2_corrected_x2(__fadd2_rn(vp[k2], mm), ch, cl);
+            const float2 xx =
+                __ffma2_rn(al2, e, __fmul2_rn(nb2, make_float2(q[2 * k2], q[2 * k2 + 1])));
+            t[2 * k2] = fmaxf(xx.x, 0.f);
+            t[2 * k2 + 1] = fmaxf(xx.y, 0.f);
+          }
+        } else {
+#pragma unroll
+          for (int k2 = 0; k2 < 8; ++k2)
+            t[k2] = fmaxf(fmaf(alpha1, L::exp_pass(v[k2], rowmax, c_hi, c_lo), -beta * q[k2]),
+                          0.f);
+        }
+        while (mp < nmask && mtok[mp] < xg) ++mp;
+        for (int mq = mp; mq < nmask && mtok[mq] < xg + kChunk; ++mq) {
+          const int off = mtok[mq] - xg;
+          const float mv = (kind == kJobPass) ? 0.f : mval[mq];
+#pragma unroll
+          for (int k2 = 0; k2 < 8; ++k2) if (k2 == off) t[k2] = mv;
+        }
+        if (kind == kJobPass) {
+          if (valid) acc.add(sum8(t));
+        } else {
+          const float ts = warp_sum(valid ? sum8(t) : 0.f);
+          if (lane == 0)
+            __stcg(f.tiles + (size_t)b * f.ntiles + (x + t0) / kTileElems, make_float2(ts, 0.f));
+        }
+      }
+    }
+    __syncwarp();
+    const bool last = (meta.flags & kStageLast) != 0;
+    if (!last) {
+      if (lane == 0) mbar_arrive(&m.empty_bar[stage]);
+    } else {
+      // ---- the slice's partial: per-warp values, combined by warp 0 ----
+      float2 mine;
+      if (kind == kJobStats) {
+        const float wm = warp_max(m_run);
+        const float part =
+            (m_run == TV_NEG_INF) ? 0.f : acc.value() * L::exp_rel(m_run, wm, c_hi, c_lo);
+        mine = make_float2(wm, warp_sum(part));
+      } else if (kind == kJobPass) {
+        mine = make_float2(warp_sum(acc.value()), 0.f);
+      } else {
+        mine = make_float2(0.f, 0.f);
+        fence_gpu();   // this warp's bonus tiles, before warp 0 reads them
+      }
+      if (lane == 0) {
+        m.sh->red[stage][wid] = mine;
+        mbar_arrive(&m.red_bar[stage]);      // release: red[] and the tiles
+        mbar_arrive(&m.slot_free[slot]);     // done with the slot's masks
+      }
+      if (wid == 0) {
+        const bool got = mbar_wait_warp(&m.red_bar[stage], (red_phase >> stage) & 1u);
+        red_phase ^= 1u << stage;
+        if (!got) {
+          if (lane == 0) raise_abort(a, f);
+          break;
+        }
+        float px = 0.f, py = 0.f;
+        if (kind == kJobStats) {
+          float M = TV_NEG_INF;
+          for (int w = 0; w < kNCW; ++w) M = fmaxf(M, m.sh->red[stage][w].x);
+          for (int w = 0; w < kNCW; ++w) {
+            const float2 r = m.sh->red[stage][w];
+            if (r.x != TV_NEG_INF) py += r.y * L::exp_rel(r.x, M, c_hi, c_lo);
+          }
+          px = M;
+        } else if (kind == kJobPass) {
+          for (int w = 0; w < kNCW; ++w) px += m.sh->red[stage][w].x;
+        } else {
+          // bonus: the slice's total (leaf: relative to the slice's own max)
+          fence_gpu();
+          const int t_lo = x0 / kTileElems, t_hi = (x1 + kTileElems - 1) / kTileElems;
+          const float2* tl = f.tiles + (size_t)b * f.ntiles;
+          if (kind == kJobBonusLeaf) {
+            float lm = TV_NEG_INF;
+            for (int k2 = t_lo + lane; k2 < t_hi; k2 += 32) lm = fmaxf(lm, __ldcg(tl + k2).y);
+            px = warp_max(lm);
+          }
+          float W = 0.f;
+          for (int k2 = t_lo + lane; k2 < t_hi; k2 += 32) {
+            const float2 tv = __ldcg(tl + k2);
+            W += (kind == kJobBonusLeaf)
+                     ? ((tv.y == TV_NEG_INF) ? 0.f : tv.x * L::exp_rel(tv.y, px, c_hi, c_lo))
+                     : tv.x;
+          }
+          py = warp_sum(W);
+          fence_gpu();   // the tiles before the partial that announces them
+        }
+        if (lane == 0) {
+          st_relaxed_u64(f.part + ((size_t)b * R + row_idx) * f.Kmax + slice, pack_part(px, py));
+          mbar_arrive(&m.empty_bar[stage]);   // only now may the stage (and red[stage]) be reused
+        }
+      } else if (lane == 0) {
+        mbar_arrive(&m.empty_bar[stage]);
+      }
+    }
+    if (++stage == n_stages) { stage = 0; phase ^= 1; }
+  }
+}
+
+// --------------------------------------------------------------- owner --
+
+// Publishes the own tree's current job (ctl.job) as slice items.
 __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const FlowArgs& f,
                          int b, int V, int lane) {
   const Job& j = sh.ctl.job;
@@ -123,6 +537,11 @@ __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const
     f.job_mtok[b * R + q] = s.mask_tok[q];
     f.job_mval[b * R + q] = s.mask_val[q];
   }
+  // the job's partial slots start as "not yet"
+  for (int q = lane; q < n; q += 32) {
+    const int r = q / K;
+    __stcg(f.part + ((size_t)b * R + r) * f.Kmax + (q - r * K), kNoPart);
+  }
   unsigned base = 0u;
   if (lane == 0) base = atomicAdd(&f.ctr[kCtrTail], (unsigned)n);
   base = __shfl_sync(0xffffffffu, base, 0);
@@ -131,11 +550,6 @@ __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const
   if ((size_t)base + n + kMaxGrid > (size_t)f.cap) {
     if (lane == 0) raise_abort(a, f);
     return;
-  }
-  // the job's partial slots start as "not yet"
-  for (int q = lane; q < n; q += 32) {
-    const int r = q / K;
-    __stcg(f.part + ((size_t)b * R + r) * f.Kmax + (q - r * K), kNoPart);
   }
   const int4 w1 = make_int4(j.kind, slice, nmask, 0);
   const int4 w2 = make_int4(__float_as_int(j.alpha1), __float_as_int(j.beta),
@@ -160,710 +574,399 @@ __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const
   }
 }
 
-// ------------------------------------------------------------- the kernel --
-
-template <typename L, int kNCW>
-__global__ void __launch_bounds__(kNCW * 32 + 32, 16 / kNCW)
-    tv_flow_kernel(TravArgs args, FlowArgs f, int n_stages) {
-  extern __shared__ __align__(128) char smem_raw[];
-  __shared__ __align__(8) uint64_t full_bar[kMaxStages];
-  __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
-  __shared__ Shared sh;
-
-  using E = typename L::elem;
-  constexpr int kConsumers = kNCW * 32;
-  constexpr int kThreads = kConsumers + 32;
-  constexpr int kWarps = kThreads / 32;
-  constexpr int kStageBytes = stage_bytes(kNCW);
-  constexpr int kSweep = kConsumers * kChunk;
-  constexpr int kLB = L::kBytes;
-  constexpr int kPairElems = kStageBytes / (kLB + 4) / kTileElems * kTileElems;
-  constexpr int kRowElems = kStageBytes / kLB;
-
-  const int R = args.N + 1, V = args.V, B = args.B;
-  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
-  const bool producer = (wid == kNCW);
-  const float c_hi = args.c_hi, c_lo = args.c_lo;
-  char* ring = smem_raw;
-  TreeSmem s = carve_tree_nt(smem_raw + (size_t)n_stages * kStageBytes, R, 0);
-  int* it_mtok = reinterpret_cast<int*>(smem_raw + (size_t)n_stages * kStageBytes +
-                                        ((tree_smem_bytes_nt(R, 0) + 15) & ~(size_t)15));
-  float* it_mval = reinterpret_cast<float*>(it_mtok + R);
-  const E* logits = reinterpret_cast<const E*>(args.logits);
-  // with fewer trees than half the CTAs, owners leave the slices to CTAs
-  // without a tree so that their own combines are never delayed
-  const bool owners_serve = 2 * B >= (int)gridDim.x;
-
-  if (tid == 0) {
-    for (int k = 0; k < n_stages; ++k) {
-      mbar_init(&full_bar[k], 1);
-      mbar_init(&empty_bar[k], kNCW);
-    }
-    fence_mbar_init();
-    sh.my_tree = -1;
+// Structure, validation and gathers of tree b; leaves ctl ready to run.
+template <typename L>
+__device__ void owner_new_tree(const TravArgs& a, const TreeSmem& s, Shared& sh, int b,
+                               int lane) {
+  const int R = a.N + 1, V = a.V;
+  const size_t row0 = (size_t)b * R;
+  const typename L::elem* logits = reinterpret_cast<const typename L::elem*>(a.logits);
+  if (lane == 0) {
     sh.outstanding = 0;
-    sh.ticket = kNoTicket;
-    sh.trees_left = 1;
+    Ctl& c = sh.ctl;
+    c.bad = 0u;
+    c.accepted = -1;
+    c.node = 0;
+    c.pending = -1;
+    c.masked_sum = 0.0;
+    c.n_tests = c.n_passes = 0;
+    c.job.kind = 0;
   }
-  __syncthreads();
-
-  int stage = 0, phase = 0;   // ring position (producer and consumers alike)
-  unsigned long long idle_since = 0ull;
-  unsigned polls = 0u, nap = 32u;
-  for (;;) {
-    // ---------------- warp 0 decides what this CTA does next ----------------
-    if (wid == 0) {
-      const int mt = sh.my_tree;
-      // the own job is finished when none of its partial slots is "not yet";
-      // the lanes poll them, keeping what they read for the combine
-      bool job_done = false;
-      const int nout = sh.outstanding;
-      if (mt >= 0 && nout > 0) {
-        const int K = sh.jK;
-        bool all = true;
-        for (int q = lane; q < nout; q += 32) {
-          const int r = q / K;
-          const unsigned long long v =
-              ld_relaxed_u64(f.part + ((size_t)mt * R + r) * f.Kmax + (q - r * K));
-          if (v == kNoPart) all = false;
-          else if (q < kPBuf) sh.pbuf[q] = unpack_part(v);
-        }
-        job_done = __all_sync(0xffffffffu, all);
-      }
-      if (lane == 0) {
-        // Polls touch only this CTA's ticket slot and its own tree's partials;
-        // the shared abort flag is read every 32nd round, the shared counters
-        // only when about to take a new tree or ticket.
-        int act = kActIdle;
-        const unsigned h = sh.ticket;
-        const unsigned long long want = (f.epoch << 32) | (unsigned long long)h;
-        const unsigned long long tag =
-            (h < (unsigned)f.cap) ? ld_relaxed_u64(&f.items[h].tag) : 0ull;
-        const unsigned abort_f = ((++polls & 31u) == 0u) ? ld_relaxed_u32(&f.ctr[kCtrAbort]) : 0u;
-        if (abort_f) {
-          act = kActExit;
-        } else if (job_done) {
-          // the bonus draw reads tiles written before its partials
-          if (sh.jkind == kJobBonusLeaf || sh.jkind == kJobBonusRes) fence_gpu();
-          act = kActCombine;
-        } else if (h < (unsigned)f.cap && tag == want) {
-          fence_gpu();
-          const int4* bp = reinterpret_cast<const int4*>(f.items + h);
-          sh.it[0] = __ldcg(bp);
-          sh.it[1] = __ldcg(bp + 1);
-          sh.it[2] = __ldcg(bp + 2);
-          sh.ticket = kNoTicket;
-          act = kActItem;
-        } else if (h < (unsigned)f.cap && tag == (want | kExitTag)) {
-          act = kActExit;   // every tree is done
-        } else {
-          if (mt < 0 && sh.trees_left) {
-            if (ld_relaxed_u32(&f.ctr[kCtrNextTree]) < (unsigned)B) {
-              const unsigned t = atomicAdd(&f.ctr[kCtrNextTree], 1u);
-              if (t < (unsigned)B) {
-                sh.my_tree = (int)t;
-                act = kActNewTree;
-              } else {
-                sh.trees_left = 0;
-              }
-            } else {
-              sh.trees_left = 0;
-            }
-          }
-          if (act == kActIdle && h == kNoTicket && (mt < 0 || owners_serve)) {
-            if (ld_relaxed_u32(&f.ctr[kCtrDone]) >= (unsigned)B)
-              act = kActExit;   // nothing will be posted any more
-            else
-              sh.ticket = atomicAdd(&f.ctr[kCtrHead], 1u);   // polled from the next round on
-          }
-        }
-        if (act == kActIdle) {
-          const unsigned long long now = global_ns();
-          if (idle_since == 0ull) {
-            idle_since = now;
-          } else if (now - idle_since > kIdleNs) {   // no progress for seconds: give up cleanly
-            raise_abort(args, f);
-            act = kActExit;
-          }
-          if (act == kActIdle) {
-            __nanosleep(nap);
-            if (nap < 256u) nap <<= 1;
-          }
-        } else {
-          idle_since = 0ull;
-          nap = 32u;
-        }
-        sh.act = act;
-      }
-    }
-    named_sync(1, kThreads);
-    const int act = sh.act;
-    if (act == kActExit) break;
-    if (act == kActIdle) continue;
-
-    if (act == kActItem) {
-      // ---------------- one slice of some tree's job ----------------
-      const int b = sh.it[0].x, node = sh.it[0].y, item_row = sh.it[0].z, item_slice = sh.it[0].w;
-      const int kind = sh.it[1].x, slice_len = sh.it[1].y, nmask = sh.it[1].z;
-      const float alpha1 = __int_as_float(sh.it[2].x);
-      const float beta = __int_as_float(sh.it[2].y);
-      const float rowmax = __int_as_float(sh.it[2].z);
-      const int x0 = item_slice * slice_len;
-      const int x1 = min(V, x0 + slice_len);
-      const size_t row = ((size_t)b * R + node) * (size_t)V;
-      const bool pair = (kind == kJobPass || kind == kJobBonusRes);
-      const int per = pair ? kPairElems : kRowElems;
-      for (int q = tid; q < nmask; q += kThreads) {
-        it_mtok[q] = __ldcg(f.job_mtok + (size_t)b * R + q);
-        it_mval[q] = __ldcg(f.job_mval + (size_t)b * R + q);
-      }
-      __syncthreads();
-      if (producer) {
-        if (lane == 0) {
-          for (int x = x0; x < x1; x += per) {
-            const int n = min(per, x1 - x);
-            if (!mbar_wait(&empty_bar[stage], phase ^ 1)) {
-              raise_abort(args, f);
-              break;
-            }
-            char* dst = ring + (size_t)stage * kStageBytes;
-            const uint32_t lbytes = (uint32_t)n * kLB;
-            const uint32_t qbytes = pair ? (uint32_t)n * 4u : 0u;
-            mbar_arrive_expect_tx(&full_bar[stage], lbytes + qbytes);
-            tma_load_1d(dst, logits + row + x, lbytes, &full_bar[stage]);
-            if (pair)
-              tma_load_1d(dst + (size_t)kPairElems * kLB, args.draft_probs + row + x, qbytes,
-                          &full_bar[stage]);
-            if (++stage == n_stages) { stage = 0; phase ^= 1; }
-          }
-        }
-        stage = __shfl_sync(0xffffffffu, stage, 0);
-        phase = __shfl_sync(0xffffffffu, phase, 0);
-      } else {
-        float m_run = TV_NEG_INF;
-        Comp acc;
-        int mp = 0;
-        const float2 ch = make_float2(c_hi, c_hi), cl = make_float2(c_lo, c_lo);
-        bool fail = false;
-        for (int x = x0; x < x1; x += per) {
-          const int n = min(per, x1 - x);
-          // every issued copy is waited for (bounded), even after a failure
-          if (!mbar_wait(&full_bar[stage], phase)) fail = true;
-          if (!fail) {
-            const char* buf = ring + (size_t)stage * kStageBytes;
-            const E* lb = reinterpret_cast<const E*>(buf);
-            const float* qb = reinterpret_cast<const float*>(buf + (size_t)kPairElems * kLB);
-            for (int t0 = wid * kTileElems; t0 < n; t0 += kSweep) {
-              const int e0 = t0 + lane * kChunk;
-              const bool valid = e0 < n;
-              const int xg = x + e0;
-              float v[8];
-              float2 vp[4];
-              if constexpr (kLB == 2) {
-                if (valid) bf16x8_pairs(lds128(lb + e0), vp);
-                else {
-#pragma unroll
-                  for (int k2 = 0; k2 < 4; ++k2) vp[k2] = make_float2(-9984.f, -9984.f);
-                }
-#pragma unroll
-                for (int k2 = 0; k2 < 4; ++k2) { v[2 * k2] = vp[k2].x; v[2 * k2 + 1] = vp[k2].y; }
-              } else {
-                if (valid) {
-                  const uint4 a4 = lds128(lb + e0);
-                  const uint4 b4 = lds128(lb + e0 + 4);
-                  v[0] = __uint_as_float(a4.x); v[1] = __uint_as_float(a4.y);
-                  v[2] = __uint_as_float(a4.z); v[3] = __uint_as_float(a4.w);
-                  v[4] = __uint_as_float(b4.x); v[5] = __uint_as_float(b4.y);
-                  v[6] = __uint_as_float(b4.z); v[7] = __uint_as_float(b4.w);
-                } else {
-#pragma unroll
-                  for (int k2 = 0; k2 < 8; ++k2) v[k2] = TV_NEG_INF;
-                }
-              }
-              if (kind == kJobStats) {
-                if (valid) {
-                  float cm = v[0];
-#pragma unroll
-                  for (int k2 = 1; k2 < 8; ++k2) cm = fmaxf(cm, v[k2]);
-                  if (cm > m_run) {
-                    if (m_run != TV_NEG_INF) {
-                      const float sc = L::exp_rel(m_run, cm, c_hi, c_lo);
-                      acc.s *= sc;
-                      acc.c *= sc;
-                    }
-                    m_run = cm;
-                  }
-                  float sum;
-                  if constexpr (kLB == 2) {
-                    const float2 mm = make_float2(-m_run, -m_run);
-                    float2 e[4];
-#pragma unroll
-                    for (int k2 = 0; k2 < 4; ++k2) e[k2] = exp2_split_x2(__fadd2_rn(vp[k2], mm), ch, cl);
-                    const float2 s2 = __fadd2_rn(__fadd2_rn(e[0], e[1]), __fadd2_rn(e[2], e[3]));
-                    sum = s2.x + s2.y;
-                  } else {
-                    float t[8];
-#pragma unroll
-                    for (int k2 = 0; k2 < 8; ++k2) t[k2] = L::exp_rel(v[k2], m_run, c_hi, c_lo);
-                    sum = sum8(t);
-                  }
-                  acc.add(sum);
-                }
-              } else if (kind == kJobBonusLeaf) {
-                float lm = v[0];
-#pragma unroll
-                for (int k2 = 1; k2 < 8; ++k2) lm = fmaxf(lm, v[k2]);
-                const float tm = warp_max(lm);
-                float t[8];
-#pragma unroll
-                for (int k2 = 0; k2 < 8; ++k2) t[k2] = L::exp_pass(v[k2], tm, c_hi, c_lo);
-                const float ts = warp_sum(valid ? sum8(t) : 0.f);
-                if (lane == 0)
-                  __stcg(f.tiles + (size_t)b * f.ntiles + (x + t0) / kTileElems,
-                         make_float2(ts, tm));
-              } else {
-                float q[8];
-                if (valid) {
-                  const uint4 qa = lds128(qb + e0);
-                  const uint4 qc = lds128(qb + e0 + 4);
-                  q[0] = __uint_as_float(qa.x); q[1] = __uint_as_float(qa.y);
-                  q[2] = __uint_as_float(qa.z); q[3] = __uint_as_float(qa.w);
-                  q[4] = __uint_as_float(qc.x); q[5] = __uint_as_float(qc.y);
-                  q[6] = __uint_as_float(qc.z); q[7] = __uint_as_float(qc.w);
-                } else {
-#pragma unroll
-                  for (int k2 = 0; k2 < 8; ++k2) q[k2] = 0.f;
-                }
-                float t[8];
-                if constexpr (kLB == 2) {
-                  const float2 mm = make_float2(-rowmax, -rowmax);
-                  const float2 al2 = make_float2(alpha1, alpha1);
-                  const float2 nb2 = make_float2(-beta, -beta);
-#pragma unroll
-                  for (int k2 = 0; k2 < 4; ++k2) {
-                    const float2 e = exp2_corrected_x2(__fadd2_rn(vp[k2], mm), ch, cl);
-                    const float2 xx = __ffma2_rn(al2, e, __fmul2_rn(nb2, make_float2(q[2 * k2], q[2 * k2 + 1])));
-                    t[2 * k2] = fmaxf(xx.x, 0.f);
-                    t[2 * k2 + 1] = fmaxf(xx.y, 0.f);
-                  }
-                } else {
-#pragma unroll
-                  for (int k2 = 0; k2 < 8; ++k2)
-                    t[k2] = fmaxf(fmaf(alpha1, L::exp_pass(v[k2], rowmax, c_hi, c_lo),
-                                       -beta * q[k2]), 0.f);
-                }
-                while (mp < nmask && it_mtok[mp] < xg) ++mp;
-                for (int mq = mp; mq < nmask && it_mtok[mq] < xg + kChunk; ++mq) {
-                  const int off = it_mtok[mq] - xg;
-                  const float mv = (kind == kJobPass) ? 0.f : it_mval[mq];
-#pragma unroll
-                  for (int k2 = 0; k2 < 8; ++k2) if (k2 == off) t[k2] = mv;
-                }
-                if (kind == kJobPass) {
-                  if (valid) acc.add(sum8(t));
-                } else {
-                  const float ts = warp_sum(valid ? sum8(t) : 0.f);
-                  if (lane == 0)
-                    __stcg(f.tiles + (size_t)b * f.ntiles + (x + t0) / kTileElems,
-                           make_float2(ts, 0.f));
-                }
-              }
-            }
-          }
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&empty_bar[stage]);
-          if (++stage == n_stages) { stage = 0; phase ^= 1; }
-        }
-        if (fail) raise_abort(args, f);
-        // ---- the slice's partial result ----
-        if (kind == kJobStats) {
-          const float wm = warp_max(m_run);
-          if (lane == 0) sh.red_a[wid] = wm;
-          named_sync(2, kConsumers);
-          float M = sh.red_a[0];
-#pragma unroll
-          for (int w = 1; w < kNCW; ++w) M = fmaxf(M, sh.red_a[w]);
-          float part = (m_run == TV_NEG_INF) ? 0.f : acc.value() * L::exp_rel(m_run, M, c_hi, c_lo);
-          part = warp_sum(part);
-          if (lane == 0) sh.red_b[wid] = part;
-          named_sync(2, kConsumers);
-          if (tid == 0) {
-            float S = 0.f;
-            for (int w = 0; w < kNCW; ++w) S += sh.red_b[w];
-            sh.out_x = M;
-            sh.out_y = S;
-          }
-        } else if (kind == kJobPass) {
-          const float ws = warp_sum(acc.value());
-          if (lane == 0) sh.red_a[wid] = ws;
-          named_sync(2, kConsumers);
-          if (tid == 0) {
-            float S = 0.f;
-            for (int w = 0; w < kNCW; ++w) S += sh.red_a[w];
-            sh.out_x = S;
-            sh.out_y = 0.f;
-          }
-        } else {
-          // bonus: the slice's total (leaf: relative to the slice's own max),
-          // from the tiles this CTA just wrote
-          fence_gpu();
-          named_sync(2, kConsumers);
-          if (wid == 0) {
-            const int t_lo = x0 / kTileElems, t_hi = (x1 + kTileElems - 1) / kTileElems;
-            const float2* tl = f.tiles + (size_t)b * f.ntiles;
-            float Mc = 0.f;
-            if (kind == kJobBonusLeaf) {
-              float lm = TV_NEG_INF;
-              for (int k2 = t_lo + lane; k2 < t_hi; k2 += 32) lm = fmaxf(lm, __ldcg(tl + k2).y);
-              Mc = warp_max(lm);
-            }
-            float W = 0.f;
-            for (int k2 = t_lo + lane; k2 < t_hi; k2 += 32) {
-              const float2 tv = __ldcg(tl + k2);
-              W += (kind == kJobBonusLeaf)
-                       ? ((tv.y == TV_NEG_INF) ? 0.f : tv.x * L::exp_rel(tv.y, Mc, c_hi, c_lo))
-                       : tv.x;
-            }
-            W = warp_sum(W);
-            if (lane == 0) {
-              sh.out_x = Mc;
-              sh.out_y = W;
-            }
-          }
-        }
-      }
-      named_sync(1, kThreads);
-      if (tid == 0)   // the partial is its own completion flag
-        st_relaxed_u64(f.part + ((size_t)b * R + item_row) * f.Kmax + item_slice,
-                       pack_part(sh.out_x, sh.out_y));
-      continue;
-    }
-
-    const int b = sh.my_tree;
-    const size_t row0 = (size_t)b * R;
-    if (act == kActNewTree) {
-      // ---------------- a new tree: structure, validation, gathers ----------------
-      if (tid == 0) {
-        sh.outstanding = 0;
-        Ctl& c = sh.ctl;
-        c.bad = 0u;
-        c.accepted = -1;
-        c.node = 0;
-        c.pending = -1;
-        c.masked_sum = 0.0;
-        c.n_tests = c.n_passes = 0;
-        c.job.kind = 0;
-      }
-      for (int i = tid; i < R; i += kThreads) {
-        s.par[i] = args.parents[row0 + i];
-        s.tok[i] = args.tokens[row0 + i];
-        s.first[i] = 0x7fffffff;
-        s.npass[i] = 0;
-        s.state[i] = kAlive;
-        s.a[i] = 1.0;
-        s.b[i] = 0.0;
-        s.Z[i] = 1.0;
-        s.invZ[i] = 1.0;
-        s.m[i] = 0.0;
-        s.p[i] = 0.0;
-        s.rows[i] = 0.f;
-        s.dbgp[i] = __int_as_float(0x7fc00000);
-      }
-      __syncthreads();
-      {
-        uint32_t bad = 0u;
-        for (int i = tid; i < R; i += kThreads) {
-          const int p = s.par[i];
-          if (i == 0) {
-            if (p != -1) bad |= 1u;
-          } else {
-            if (p < 0 || p >= i) bad |= 1u;
-            else atomicMin(&s.first[p], i);
-            const int t = s.tok[i];
-            if (t < 0 || t >= V) bad |= 2u;
-          }
-        }
-        if (bad) atomicOr(&sh.ctl.bad, bad);
-      }
-      __syncthreads();
-      if (sh.ctl.bad == 0u) {
-        uint32_t bad = 0u;
-        for (int i = tid; i < R; i += kThreads) {
-          if (s.first[i] == 0x7fffffff) s.first[i] = -1;
-          int nx = -1;
-          if (i > 0) {
-            const int p = s.par[i], t = s.tok[i];
-            for (int j = i + 1; j < R; ++j) {
-              if (s.par[j] != p) continue;
-              if (nx < 0) nx = j;
-              if (s.tok[j] == t) bad |= 4u;
-            }
-            const size_t prow = (row0 + p) * (size_t)V;
-            s.gl[i] = L::at(logits + prow, t);
-            s.gq[i] = __ldg(args.draft_probs + prow + t);
-            if (!(s.gq[i] > 0.f)) bad |= 8u;
-            s.invq[i] = 1.0 / (double)s.gq[i];
-          }
-          s.next[i] = nx;
-        }
-        if (bad) atomicOr(&sh.ctl.bad, bad);
-      }
-      __syncthreads();
-      if (tid == 0) {
-        if (sh.ctl.bad == 0u) {
-          s.p[0] = 1.0;
-          control_step(s, sh.ctl, args.uniforms + row0 + b);
-        } else {
-          sh.ctl.job.kind = kJobDone;
-        }
-      }
+  for (int i = lane; i < R; i += 32) {
+    s.par[i] = a.parents[row0 + i];
+    s.tok[i] = a.tokens[row0 + i];
+    s.first[i] = 0x7fffffff;
+    s.npass[i] = 0;
+    s.state[i] = kAlive;
+    s.a[i] = 1.0;
+    s.b[i] = 0.0;
+    s.Z[i] = 1.0;
+    s.invZ[i] = 1.0;
+    s.m[i] = 0.0;
+    s.p[i] = 0.0;
+    s.rows[i] = 0.f;
+    s.dbgp[i] = __int_as_float(0x7fc00000);
+  }
+  __syncwarp();
+  uint32_t bad = 0u;
+  for (int i = lane; i < R; i += 32) {
+    const int p = s.par[i];
+    if (i == 0) {
+      if (p != -1) bad |= 1u;
     } else {
-      // ---------------- kActCombine: own tree's job finished; combine, advance ----------------
-      const int K = sh.jK;
-      const bool in_smem = sh.outstanding <= kPBuf;
-      auto part_of = [&](int r, int k) -> float2 {
-        return in_smem ? sh.pbuf[r * K + k]
-                       : unpack_part(__ldcg(f.part + (row0 + r) * f.Kmax + k));
-      };
-      if (sh.jkind == kJobStats) {
-        // one warp per row: normaliser from the slices, then the children's M_b0
-        for (int r = wid; r < sh.jrows; r += kWarps) {
-          float M = TV_NEG_INF;
-          for (int k2 = lane; k2 < K; k2 += 32) M = fmaxf(M, part_of(r, k2).x);
-          M = warp_max(M);
-          float S = 0.f;
-          for (int k2 = lane; k2 < K; k2 += 32) {
-            const float2 pk = part_of(r, k2);
-            if (pk.x != TV_NEG_INF) S += pk.y * L::exp_rel(pk.x, M, c_hi, c_lo);
-          }
-          S = warp_sum(S);
-          const int node = s.job_rows[r];
-          if (lane == 0) {
-            s.rowm[node] = M;
-            s.rows[node] = S;
-            s.invs[node] = 1.0 / (double)S;
-            if (!(S > 0.f)) atomicOr(&sh.ctl.bad, 64u);
-          }
-          __syncwarp();
-          children_mb0(s, node, args.c, lane);
+      if (p < 0 || p >= i) bad |= 1u;
+      else atomicMin(&s.first[p], i);
+      const int t = s.tok[i];
+      if (t < 0 || t >= V) bad |= 2u;
+    }
+  }
+  bad = __reduce_or_sync(0xffffffffu, bad);
+  __syncwarp();
+  if (bad == 0u) {
+    uint32_t bad2 = 0u;
+    for (int i = lane; i < R; i += 32) {
+      if (s.first[i] == 0x7fffffff) s.first[i] = -1;
+      int nx = -1;
+      if (i > 0) {
+        const int p = s.par[i], t = s.tok[i];
+        for (int j = i + 1; j < R; ++j) {
+          if (s.par[j] != p) continue;
+          if (nx < 0) nx = j;
+          if (s.tok[j] == t) bad2 |= 4u;
         }
-      } else if (sh.jkind == kJobPass) {
-        if (wid == 0) {
-          float S = 0.f;
-          for (int k2 = lane; k2 < K; k2 += 32) S += part_of(0, k2).x;
-          S = warp_sum(S);
-          if (lane == 0) sh.ctl.S = S;
-        }
-      } else if (wid == 0) {
-        // ---- bonus: crossing slice, crossing tile, token ----
-        const Job& job = sh.ctl.job;
-        const bool leaf = (sh.jkind == kJobBonusLeaf);
-        const int node = job.node;
-        const int slice_len = sh.jslice;
-        float Mg = TV_NEG_INF;
-        if (leaf) {
-          for (int k2 = lane; k2 < K; k2 += 32) Mg = fmaxf(Mg, part_of(0, k2).x);
-          Mg = warp_max(Mg);
-        }
-        auto slice_scale = [&](float mx) -> float {
-          return leaf ? ((mx == TV_NEG_INF) ? 0.f : L::exp_rel(mx, Mg, c_hi, c_lo)) : 1.f;
-        };
-        float W = 0.f;
-        for (int k2 = lane; k2 < K; k2 += 32) {
-          const float2 pk = part_of(0, k2);
-          W += pk.y * slice_scale(pk.x);
-        }
-        W = warp_sum(W);
-        const float target = args.uniforms[row0 + b + R] * W;
-        // first slice whose running total exceeds the target (warp scan per 32 slices)
-        int owner = -1, last_pos = -1;
-        float before = 0.f, scale = 0.f, last_before = 0.f, last_scale = 0.f, base = 0.f;
-        for (int k0 = 0; k0 < K && owner < 0; k0 += 32) {
-          float wk = 0.f, sk = 0.f;
-          if (k0 + lane < K) {
-            const float2 pk = part_of(0, k0 + lane);
-            sk = slice_scale(pk.x);
-            wk = pk.y * sk;
-          }
-          float v = wk;
-#pragma unroll
-          for (int o = 1; o < 32; o <<= 1) {
-            const float w2 = __shfl_up_sync(0xffffffffu, v, o);
-            if (lane >= o) v += w2;
-          }
-          const unsigned pos = __ballot_sync(0xffffffffu, wk > 0.f);
-          if (pos) {
-            const int l = 31 - __clz(pos);
-            last_pos = k0 + l;
-            last_before = base + __shfl_sync(0xffffffffu, v - wk, l);
-            last_scale = __shfl_sync(0xffffffffu, sk, l);
-          }
-          const unsigned hit = __ballot_sync(0xffffffffu, (k0 + lane < K) && (target < base + v));
-          if (hit) {
-            const int l = __ffs(hit) - 1;
-            owner = k0 + l;
-            before = base + __shfl_sync(0xffffffffu, v - wk, l);
-            scale = __shfl_sync(0xffffffffu, sk, l);
-          }
-          base += __shfl_sync(0xffffffffu, v, 31);
-        }
-        if (owner < 0) {   // rounding put the target past the total: last slice with weight
-          owner = (last_pos >= 0) ? last_pos : 0;
-          before = (last_pos >= 0) ? last_before : 0.f;
-          scale = (last_pos >= 0) ? last_scale : slice_scale(part_of(0, 0).x);
-        }
-        const float Mc = part_of(0, owner).x;
-        const float lt = (scale > 0.f) ? (target - before) / scale : 0.f;
-        // tiles of the crossing slice, in that slice's units
-        const int sx0 = owner * slice_len, sx1 = min(V, sx0 + slice_len);
-        const int t_lo = sx0 / kTileElems, t_hi = (sx1 + kTileElems - 1) / kTileElems;
-        const float2* tl = f.tiles + (size_t)b * f.ntiles;
-        auto tile_w = [&](float2 tv) -> float {
-          return leaf ? ((tv.y == TV_NEG_INF) ? 0.f : tv.x * L::exp_rel(tv.y, Mc, c_hi, c_lo))
-                      : tv.x;
-        };
-        int tile = -1, last_tile = -1;
-        float tbase = 0.f, tb = 0.f, last_tbase = 0.f;
-        for (int k0 = t_lo; k0 < t_hi && tile < 0; k0 += 32) {
-          const float own = (k0 + lane < t_hi) ? tile_w(__ldcg(tl + k0 + lane)) : 0.f;
-          float v = own;
-#pragma unroll
-          for (int o = 1; o < 32; o <<= 1) {
-            const float w2 = __shfl_up_sync(0xffffffffu, v, o);
-            if (lane >= o) v += w2;
-          }
-          const unsigned pos = __ballot_sync(0xffffffffu, own > 0.f);
-          if (pos) {
-            const int l = 31 - __clz(pos);
-            last_tile = k0 + l;
-            last_tbase = tb + __shfl_sync(0xffffffffu, v - own, l);
-          }
-          const unsigned hit = __ballot_sync(0xffffffffu, (k0 + lane < t_hi) && (lt < tb + v));
-          if (hit) {
-            const int l = __ffs(hit) - 1;
-            tile = k0 + l;
-            tbase = tb + __shfl_sync(0xffffffffu, v - own, l);
-          }
-          tb += __shfl_sync(0xffffffffu, v, 31);
-        }
-        if (tile < 0) {
-          tile = (last_tile >= 0) ? last_tile : t_lo;
-          tbase = (last_tile >= 0) ? last_tbase : 0.f;
-        }
-        const int xs = tile * kTileElems + lane * kChunk;
-        const size_t rowoff = (row0 + node) * (size_t)V;
-        float w[8];
-        if (leaf) {
-          float v[8];
-          if (xs < sx1) load_logits<L, true>(logits + rowoff, xs, V, v);
-          else {
-#pragma unroll
-            for (int e = 0; e < 8; ++e) v[e] = TV_NEG_INF;
-          }
-#pragma unroll
-          for (int e = 0; e < 8; ++e)
-            w[e] = (v[e] == TV_NEG_INF) ? 0.f : L::exp_pass(v[e], Mc, c_hi, c_lo);
-        } else {
-          float v[8], q[8];
-          if (xs < sx1) {
-            load_logits<L, true>(logits + rowoff, xs, V, v);
-            load_probs<true>(args.draft_probs + rowoff, xs, V, q);
-          } else {
-#pragma unroll
-            for (int e = 0; e < 8; ++e) { v[e] = TV_NEG_INF; q[e] = 0.f; }
-          }
-#pragma unroll
-          for (int e = 0; e < 8; ++e)
-            w[e] = (v[e] == TV_NEG_INF) ? 0.f
-                   : fmaxf(fmaf(job.alpha1, L::exp_pass(v[e], job.rowmax, c_hi, c_lo),
-                                -job.beta * q[e]), 0.f);
-          for (int mq = 0; mq < job.nmask; ++mq) {
-            const int off = s.mask_tok[mq] - xs;
-            const float mv = s.mask_val[mq];
-#pragma unroll
-            for (int e = 0; e < 8; ++e) if (e == off) w[e] = mv;
-          }
-        }
-        float pre[8];
-        float run = 0.f;
-#pragma unroll
-        for (int e = 0; e < 8; ++e) { run += w[e]; pre[e] = run; }
-        float v = run;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const float w2 = __shfl_up_sync(0xffffffffu, v, o);
-          if (lane >= o) v += w2;
-        }
-        const float lbase = tbase + (v - run);
-        int found = 8;
-#pragma unroll
-        for (int e = 7; e >= 0; --e) if (lt < lbase + pre[e]) found = e;
-        const unsigned hit = __ballot_sync(0xffffffffu, found < 8);
-        int yy;
-        if (hit) {
-          const int l = __ffs(hit) - 1;
-          yy = tile * kTileElems + l * kChunk + __shfl_sync(0xffffffffu, found, l);
-        } else {
-          int last = -1;
-#pragma unroll
-          for (int e = 0; e < 8; ++e) if (w[e] > 0.f) last = xs + e;
-          const unsigned any = __ballot_sync(0xffffffffu, last >= 0);
-          yy = any ? __shfl_sync(0xffffffffu, last, 31 - __clz(any)) : sx1 - 1;
-        }
-        if (lane == 0) {
-          args.out_bonus[b] = yy;
-          sh.ctl.job.kind = kJobDone;
-        }
+        const size_t prow = (row0 + p) * (size_t)V;
+        s.gl[i] = L::at(logits + prow, t);
+        s.gq[i] = __ldg(a.draft_probs + prow + t);
+        if (!(s.gq[i] > 0.f)) bad2 |= 8u;
+        s.invq[i] = 1.0 / (double)s.gq[i];
       }
-      __syncthreads();
-      if (tid == 0 && sh.ctl.job.kind != kJobDone) {
-        if (sh.ctl.bad & 64u) sh.ctl.job.kind = kJobDone;
-        else control_step(s, sh.ctl, args.uniforms + row0 + b);
+      s.next[i] = nx;
+    }
+    bad = __reduce_or_sync(0xffffffffu, bad2);
+  }
+  __syncwarp();
+  if (lane == 0) {
+    sh.ctl.bad = bad;
+    if (bad == 0u) {
+      s.p[0] = 1.0;
+      control_step(s, sh.ctl, a.uniforms + row0 + b);
+    } else {
+      sh.ctl.job.kind = kJobDone;
+    }
+  }
+  __syncwarp();
+}
+
+// Combines the finished job's partials (sh.pbuf or global) and advances.
+template <typename L>
+__device__ void owner_combine(const TravArgs& a, const FlowArgs& f, const TreeSmem& s,
+                              Shared& sh, int b, int lane) {
+  const int R = a.N + 1, V = a.V;
+  const size_t row0 = (size_t)b * R;
+  const float c_hi = a.c_hi, c_lo = a.c_lo;
+  const typename L::elem* logits = reinterpret_cast<const typename L::elem*>(a.logits);
+  const int K = sh.jK;
+  const bool in_smem = sh.outstanding <= kPBuf;
+  auto part_of = [&](int r, int k) -> float2 {
+    return in_smem ? sh.pbuf[r * K + k]
+                   : unpack_part(__ldcg(f.part + (row0 + r) * f.Kmax + k));
+  };
+  if (sh.jkind == kJobStats) {
+    // normaliser of each row from its slices, then its children's M_b0
+    for (int r = 0; r < sh.jrows; ++r) {
+      float M = TV_NEG_INF;
+      for (int k2 = lane; k2 < K; k2 += 32) M = fmaxf(M, part_of(r, k2).x);
+      M = warp_max(M);
+      float S = 0.f;
+      for (int k2 = lane; k2 < K; k2 += 32) {
+        const float2 pk = part_of(r, k2);
+        if (pk.x != TV_NEG_INF) S += pk.y * L::exp_rel(pk.x, M, c_hi, c_lo);
+      }
+      S = warp_sum(S);
+      const int node = s.job_rows[r];
+      if (lane == 0) {
+        s.rowm[node] = M;
+        s.rows[node] = S;
+        s.invs[node] = 1.0 / (double)S;
+        if (!(S > 0.f)) sh.ctl.bad |= 64u;
+      }
+      __syncwarp();
+      children_mb0(s, node, a.c, lane);
+      __syncwarp();
+    }
+  } else if (sh.jkind == kJobPass) {
+    float S = 0.f;
+    for (int k2 = lane; k2 < K; k2 += 32) S += part_of(0, k2).x;
+    S = warp_sum(S);
+    if (lane == 0) sh.ctl.S = S;
+  } else {
+    // ---- bonus: crossing slice, crossing tile, token ----
+    const Job& job = sh.ctl.job;
+    const bool leaf = (sh.jkind == kJobBonusLeaf);
+    const int node = job.node;
+    const int slice_len = sh.jslice;
+    float Mg = TV_NEG_INF;
+    if (leaf) {
+      for (int k2 = lane; k2 < K; k2 += 32) Mg = fmaxf(Mg, part_of(0, k2).x);
+      Mg = warp_max(Mg);
+    }
+    auto slice_scale = [&](float mx) -> float {
+      return leaf ? ((mx == TV_NEG_INF) ? 0.f : L::exp_rel(mx, Mg, c_hi, c_lo)) : 1.f;
+    };
+    float W = 0.f;
+    for (int k2 = lane; k2 < K; k2 += 32) {
+      const float2 pk = part_of(0, k2);
+      W += pk.y * slice_scale(pk.x);
+    }
+    W = warp_sum(W);
+    const float target = a.uniforms[row0 + b + R] * W;
+    // first slice whose running total exceeds the target (warp scan per 32 slices)
+    int owner = -1, last_pos = -1;
+    float before = 0.f, scale = 0.f, last_before = 0.f, last_scale = 0.f, base = 0.f;
+    for (int k0 = 0; k0 < K && owner < 0; k0 += 32) {
+      float wk = 0.f, sk = 0.f;
+      if (k0 + lane < K) {
+        const float2 pk = part_of(0, k0 + lane);
+        sk = slice_scale(pk.x);
+        wk = pk.y * sk;
+      }
+      float v = wk;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const float w2 = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += w2;
+      }
+      const unsigned pos = __ballot_sync(0xffffffffu, wk > 0.f);
+      if (pos) {
+        const int l = 31 - __clz(pos);
+        last_pos = k0 + l;
+        last_before = base + __shfl_sync(0xffffffffu, v - wk, l);
+        last_scale = __shfl_sync(0xffffffffu, sk, l);
+      }
+      const unsigned hit = __ballot_sync(0xffffffffu, (k0 + lane < K) && (target < base + v));
+      if (hit) {
+        const int l = __ffs(hit) - 1;
+        owner = k0 + l;
+        before = base + __shfl_sync(0xffffffffu, v - wk, l);
+        scale = __shfl_sync(0xffffffffu, sk, l);
+      }
+      base += __shfl_sync(0xffffffffu, v, 31);
+    }
+    if (owner < 0) {   // rounding put the target past the total: last slice with weight
+      owner = (last_pos >= 0) ? last_pos : 0;
+      before = (last_pos >= 0) ? last_before : 0.f;
+      scale = (last_pos >= 0) ? last_scale : slice_scale(part_of(0, 0).x);
+    }
+    const float Mc = part_of(0, owner).x;
+    const float lt = (scale > 0.f) ? (target - before) / scale : 0.f;
+    // tiles of the crossing slice, in that slice's units
+    const int sx0 = owner * slice_len, sx1 = min(V, sx0 + slice_len);
+    const int t_lo = sx0 / kTileElems, t_hi = (sx1 + kTileElems - 1) / kTileElems;
+    const float2* tl = f.tiles + (size_t)b * f.ntiles;
+    auto tile_w = [&](float2 tv) -> float {
+      return leaf ? ((tv.y == TV_NEG_INF) ? 0.f : tv.x * L::exp_rel(tv.y, Mc, c_hi, c_lo))
+                  : tv.x;
+    };
+    int tile = -1, last_tile = -1;
+    float tbase = 0.f, tb = 0.f, last_tbase = 0.f;
+    for (int k0 = t_lo; k0 < t_hi && tile < 0; k0 += 32) {
+      const float own = (k0 + lane < t_hi) ? tile_w(__ldcg(tl + k0 + lane)) : 0.f;
+      float v = own;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const float w2 = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += w2;
+      }
+      const unsigned pos = __ballot_sync(0xffffffffu, own > 0.f);
+      if (pos) {
+        const int l = 31 - __clz(pos);
+        last_tile = k0 + l;
+        last_tbase = tb + __shfl_sync(0xffffffffu, v - own, l);
+      }
+      const unsigned hit = __ballot_sync(0xffffffffu, (k0 + lane < t_hi) && (lt < tb + v));
+      if (hit) {
+        const int l = __ffs(hit) - 1;
+        tile = k0 + l;
+        tbase = tb + __shfl_sync(0xffffffffu, v - own, l);
+      }
+      tb += __shfl_sync(0xffffffffu, v, 31);
+    }
+    if (tile < 0) {
+      tile = (last_tile >= 0) ? last_tile : t_lo;
+      tbase = (last_tile >= 0) ? last_tbase : 0.f;
+    }
+    const int xs = tile * kTileElems + lane * kChunk;
+    const size_t rowoff = (row0 + node) * (size_t)V;
+    float w[8];
+    if (leaf) {
+      float v[8];
+      if (xs < sx1) load_logits<L, true>(logits + rowoff, xs, V, v);
+      else {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[e] = TV_NEG_INF;
+      }
+#pragma unroll
+      for (int e = 0; e < 8; ++e)
+        w[e] = (v[e] == TV_NEG_INF) ? 0.f : L::exp_pass(v[e], Mc, c_hi, c_lo);
+    } else {
+      float v[8], q[8];
+      if (xs < sx1) {
+        load_logits<L, true>(logits + rowoff, xs, V, v);
+        load_probs<true>(a.draft_probs + rowoff, xs, V, q);
+      } else {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) { v[e] = TV_NEG_INF; q[e] = 0.f; }
+      }
+#pragma unroll
+      for (int e = 0; e < 8; ++e)
+        w[e] = (v[e] == TV_NEG_INF) ? 0.f
+               : fmaxf(fmaf(job.alpha1, L::exp_pass(v[e], job.rowmax, c_hi, c_lo),
+                            -job.beta * q[e]), 0.f);
+      for (int mq = 0; mq < job.nmask; ++mq) {
+        const int off = s.mask_tok[mq] - xs;
+        const float mv = s.mask_val[mq];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) if (e == off) w[e] = mv;
       }
     }
-    // ---------------- post the own tree's next job, or finish the tree ----------------
-    __syncthreads();
-    if (sh.ctl.job.kind == kJobDone) {
-      const bool ok = (sh.ctl.bad & (15u | 32u | 64u)) == 0u;
-      const int N = args.N;
-      for (int k2 = tid; k2 < N; k2 += kThreads) args.out_path[(size_t)b * N + k2] = -1;
-      if (args.out_node_p)
-        for (int i = tid; i < R; i += kThreads)
-          args.out_node_p[row0 + i] = ok ? s.dbgp[i] : __int_as_float(0x7fc00000);
-      __syncthreads();
-      if (tid == 0) {
-        const int acc_node = ok ? sh.ctl.accepted : -1;
-        if (acc_node >= 0) {
-          int depth = 0;
-          for (int j = acc_node; j != 0; j = s.par[j]) ++depth;
-          int k2 = depth - 1;
-          for (int j = acc_node; j != 0; j = s.par[j]) args.out_path[(size_t)b * N + (k2--)] = j;
-          args.out_accept_len[b] = depth;
-        } else {
-          args.out_accept_len[b] = -1;
-          args.out_bonus[b] = -1;
-        }
-        if (args.out_stats) {
-          int distinct = 0;
-          for (int i = 0; i < R; ++i) distinct += (s.npass[i] > 0);
-          int32_t* o = args.out_stats + (size_t)b * 4;
-          o[0] = ok ? sh.ctl.n_tests : 0;
-          o[1] = ok ? sh.ctl.n_passes : 0;
-          o[2] = ok ? distinct : 0;
-          o[3] = (acc_node >= 0 && s.first[acc_node] < 0) ? 1 : 0;
-        }
-        if (sh.ctl.bad) atomicOr(args.status, sh.ctl.bad);
-        f.finished[b] = (unsigned)f.epoch;
-        fence_gpu();
-        sh.act = (atomicAdd(&f.ctr[kCtrDone], 1u) == (unsigned)B - 1u) ? 1 : 0;
-        sh.my_tree = -1;
-        sh.outstanding = 0;
+    float pre[8];
+    float run = 0.f;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) { run += w[e]; pre[e] = run; }
+    float v = run;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float w2 = __shfl_up_sync(0xffffffffu, v, o);
+      if (lane >= o) v += w2;
+    }
+    const float lbase = tbase + (v - run);
+    int found = 8;
+#pragma unroll
+    for (int e = 7; e >= 0; --e) if (lt < lbase + pre[e]) found = e;
+    const unsigned hit = __ballot_sync(0xffffffffu, found < 8);
+    int yy;
+    if (hit) {
+      const int l = __ffs(hit) - 1;
+      yy = tile * kTileElems + l * kChunk + __shfl_sync(0xffffffffu, found, l);
+    } else {
+      int last = -1;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) if (w[e] > 0.f) last = xs + e;
+      const unsigned any = __ballot_sync(0xffffffffu, last >= 0);
+      yy = any ? __shfl_sync(0xffffffffu, last, 31 - __clz(any)) : sx1 - 1;
+    }
+    if (lane == 0) {
+      a.out_bonus[b] = yy;
+      sh.ctl.job.kind = kJobDone;
+    }
+  }
+  __syncwarp();
+  if (lane == 0 && sh.ctl.job.kind != kJobDone) {
+    if (sh.ctl.bad & 64u) sh.ctl.job.kind = kJobDone;
+    else control_step(s, sh.ctl, a.uniforms + row0 + b);
+  }
+  __syncwarp();
+}
+
+// Writes tree b's outputs; true if it was the last tree of the call.
+__device__ bool owner_finish(const TravArgs& a, const FlowArgs& f, const TreeSmem& s,
+                             Shared& sh, int b, int lane) {
+  const int R = a.N + 1, N = a.N;
+  const size_t row0 = (size_t)b * R;
+  const bool ok = (sh.ctl.bad & (15u | 32u | 64u)) == 0u;
+  for (int k2 = lane; k2 < N; k2 += 32) a.out_path[(size_t)b * N + k2] = -1;
+  if (a.out_node_p)
+    for (int i = lane; i < R; i += 32)
+      a.out_node_p[row0 + i] = ok ? s.dbgp[i] : __int_as_float(0x7fc00000);
+  __syncwarp();
+  int last = 0;
+  if (lane == 0) {
+    const int acc_node = ok ? sh.ctl.accepted : -1;
+    if (acc_node >= 0) {
+      int depth = 0;
+      for (int j = acc_node; j != 0; j = s.par[j]) ++depth;
+      int k2 = depth - 1;
+      for (int j = acc_node; j != 0; j = s.par[j]) a.out_path[(size_t)b * N + (k2--)] = j;
+      a.out_accept_len[b] = depth;
+    } else {
+      a.out_accept_len[b] = -1;
+      a.out_bonus[b] = -1;
+    }
+    if (a.out_stats) {
+      int distinct = 0;
+      for (int i = 0; i < R; ++i) distinct += (s.npass[i] > 0);
+      int32_t* o = a.out_stats + (size_t)b * 4;
+      o[0] = ok ? sh.ctl.n_tests : 0;
+      o[1] = ok ? sh.ctl.n_passes : 0;
+      o[2] = ok ? distinct : 0;
+      o[3] = (acc_node >= 0 && s.first[acc_node] < 0) ? 1 : 0;
+    }
+    if (sh.ctl.bad) atomicOr(a.status, sh.ctl.bad);
+    f.finished[b] = (unsigned)f.epoch;
+    fence_gpu();
+    last = (atomicAdd(&f.ctr[kCtrDone], 1u) == (unsigned)a.B - 1u) ? 1 : 0;
+    sh.outstanding = 0;
+  }
+  return __shfl_sync(0xffffffffu, last, 0) != 0;
+}
+
+template <typename L>
+__device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, int lane) {
+  const int R = a.N + 1, V = a.V, B = a.B;
+  Shared& sh = *m.sh;
+  const TreeSmem& s = m.s;
+  int my_tree = -1;
+  unsigned polls = 0u;
+  Backoff wait;
+  for (;;) {
+    __syncwarp();   // lane 0's updates of sh (job shape, control state) seen by all lanes
+    if (my_tree < 0) {
+      unsigned t = 0u;
+      if (lane == 0)
+        t = (ld_relaxed_u32(&f.ctr[kCtrNextTree]) < (unsigned)B)
+                ? atomicAdd(&f.ctr[kCtrNextTree], 1u) : (unsigned)B;
+      t = __shfl_sync(0xffffffffu, t, 0);
+      if (t >= (unsigned)B) break;   // no trees left for this CTA to own
+      my_tree = (int)t;
+      owner_new_tree<L>(a, s, sh, my_tree, lane);
+    } else {
+      // poll the own job's partials (kept in pbuf for the combine)
+      const int nout = sh.outstanding;
+      const int K = sh.jK;
+      bool all = true;
+      for (int q = lane; q < nout; q += 32) {
+        const int r = q / K;
+        const unsigned long long v =
+            ld_relaxed_u64(f.part + ((size_t)my_tree * R + r) * f.Kmax + (q - r * K));
+        if (v == kNoPart) all = false;
+        else if (q < kPBuf) sh.pbuf[q] = unpack_part(v);
       }
-      __syncthreads();
-      if (sh.act == 1 && wid == 0) {
-        // last tree: the tickets now held (slots from the tail up to the head)
-        // and the at most one more per CTA that may still be taken will see
-        // an exit tag instead of an item
+      const bool done = __all_sync(0xffffffffu, all);
+      if (!done) {
+        int stop = 0;
+        if (lane == 0) {
+          if ((++polls & 31u) == 0u && ld_relaxed_u32(&f.ctr[kCtrAbort])) stop = 1;
+          else if (!wait.idle()) {
+            raise_abort(a, f);
+            stop = 1;
+          }
+        }
+        if (__shfl_sync(0xffffffffu, stop, 0)) break;
+        continue;
+      }
+      wait.reset();
+      // the bonus draw reads tiles written before its partials
+      if (sh.jkind == kJobBonusLeaf || sh.jkind == kJobBonusRes) fence_gpu();
+      __syncwarp();
+      owner_combine<L>(a, f, s, sh, my_tree, lane);
+    }
+    if (sh.ctl.job.kind == kJobDone) {
+      const bool last = owner_finish(a, f, s, sh, my_tree, lane);
+      my_tree = -1;
+      if (last) {
+        // every tree is done: the tickets now held (slots from the tail up to
+        // the head) and the at most one more per CTA that may still be taken
+        // see an exit tag instead of an item
         unsigned lo = 0u, hi = 0u;
         if (lane == 0) {
           lo = atomicAdd(&f.ctr[kCtrTail], 0u);
@@ -874,16 +977,60 @@ __global__ void __launch_bounds__(kNCW * 32 + 32, 16 / kNCW)
         for (unsigned q = lo + lane; q < hi; q += 32)
           st_relaxed_u64(&f.items[q].tag, (f.epoch << 32) | q | kExitTag);
       }
-    } else if (wid == 0) {
-      post_job(s, sh, args, f, b, V, lane);
+    } else {
+      post_job(s, sh, a, f, my_tree, V, lane);
     }
   }
+}
+
+// ------------------------------------------------------------- the kernel --
+
+template <typename L, int kNCW>
+__global__ void __launch_bounds__(Shape<L, kNCW>::kThreads, 16 / kNCW)
+    tv_flow_kernel(TravArgs args, FlowArgs f, int n_stages) {
+  using S = Shape<L, kNCW>;
+  extern __shared__ __align__(128) char smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[kMaxStages];
+  __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
+  __shared__ __align__(8) uint64_t red_bar[kMaxStages];
+  __shared__ __align__(8) uint64_t slot_free[kSlots];
+  __shared__ Shared sh;
+
+  const int R = args.N + 1;
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  Smem m;
+  m.ring = smem_raw;
+  char* tree_base = smem_raw + (size_t)n_stages * S::kStageBytes;
+  m.s = carve_tree_nt(tree_base, R, 0);
+  m.mtok = reinterpret_cast<int*>(tree_base + ((tree_smem_bytes_nt(R, 0) + 15) & ~(size_t)15));
+  m.mval = reinterpret_cast<float*>(m.mtok + kSlots * R);
+  m.full_bar = full_bar;
+  m.empty_bar = empty_bar;
+  m.slot_free = slot_free;
+  m.red_bar = red_bar;
+  m.sh = &sh;
+
+  if (tid == 0) {
+    for (int k = 0; k < n_stages; ++k) {
+      mbar_init(&full_bar[k], 1);
+      mbar_init(&empty_bar[k], kNCW);
+      mbar_init(&red_bar[k], kNCW);
+    }
+    for (int k = 0; k < kSlots; ++k) mbar_init(&slot_free[k], kNCW);
+    fence_mbar_init();
+    sh.outstanding = 0;
+  }
+  __syncthreads();
+
+  if (wid < kNCW) consumer_role<L, kNCW>(args, f, m, n_stages, wid, lane);
+  else if (wid == kNCW) producer_role<L, kNCW>(args, f, m, n_stages, lane);
+  else owner_role<L>(args, f, m, lane);
 
   // ---------------- exit ----------------
   __syncthreads();
   if (ld_relaxed_u32(&f.ctr[kCtrAbort])) {
     // after an abort, trees that did not finish report "invalid"
-    for (int b = blockIdx.x * kThreads + tid; b < B; b += gridDim.x * kThreads) {
+    for (int b = blockIdx.x * S::kThreads + tid; b < args.B; b += gridDim.x * S::kThreads) {
       if (ld_relaxed_u32(&f.finished[b]) != (unsigned)f.epoch) {
         args.out_accept_len[b] = -1;
         args.out_bonus[b] = -1;
@@ -914,7 +1061,7 @@ FlowLayout flow_layout(int B, int R, int V, int min_slice) {
   FlowLayout l;
   l.kmax = (size_t)((V + min_slice - 1) / min_slice);
   // per tree: at most R rows normalised and at most R - 1 passes plus the
-  // bonus draw, each at most kmax slices
+  // bonus draw, each at most kmax slices; then room for the exit tags
   l.cap = (size_t)B * (2 * (size_t)R + 1) * l.kmax + tvk::flow::kMaxGrid;
   l.ntiles = (size_t)((V + tvk::fused::kTileElems - 1) / tvk::fused::kTileElems);
   return l;
@@ -924,7 +1071,8 @@ size_t up256(size_t n) { return (n + 255) & ~static_cast<size_t>(255); }
 
 size_t flow_smem_bytes(int R, int ncw, int stages) {
   return (size_t)stages * tvk::fused::stage_bytes(ncw) +
-         ((tvk::fused::tree_smem_bytes_nt(R, 0) + 15) & ~(size_t)15) + (size_t)R * 8 + 64;
+         ((tvk::fused::tree_smem_bytes_nt(R, 0) + 15) & ~(size_t)15) +
+         (size_t)tvk::flow::kSlots * R * 8 + 64;
 }
 
 }  // namespace
@@ -974,13 +1122,13 @@ FlowPlan tv_flow_plan(int R, int smem_per_sm, int smem_per_block, int force_ncw,
   } else {
     p.stages = 2;
     for (int st = tvk::fused::kMaxStages; st >= 2; --st)
-      if ((size_t)per_sm * (flow_smem_bytes(R, p.ncw, st) + 2048) <= (size_t)smem_per_sm) {
+      if ((size_t)per_sm * (flow_smem_bytes(R, p.ncw, st) + 4096) <= (size_t)smem_per_sm) {
         p.stages = st;
         break;
       }
   }
   p.smem = flow_smem_bytes(R, p.ncw, p.stages);
-  p.ok = p.smem + 2048 <= (size_t)smem_per_block;
+  p.ok = p.smem + 4096 <= (size_t)smem_per_block;
   return p;
 }
 
@@ -1014,11 +1162,11 @@ int tv_launch_flow(const TravArgs& a, FlowArgs f, int logit_is_bf16, const FlowP
   };
   int rc;
   if (plan.ncw == 8)
-    rc = logit_is_bf16 ? run(tv_flow_kernel<tvk::Bf16Logits, 8>, 288)
-                       : run(tv_flow_kernel<tvk::F32Logits, 8>, 288);
+    rc = logit_is_bf16 ? run(tv_flow_kernel<tvk::Bf16Logits, 8>, Shape<tvk::Bf16Logits, 8>::kThreads)
+                       : run(tv_flow_kernel<tvk::F32Logits, 8>, Shape<tvk::F32Logits, 8>::kThreads);
   else
-    rc = logit_is_bf16 ? run(tv_flow_kernel<tvk::Bf16Logits, 4>, 160)
-                       : run(tv_flow_kernel<tvk::F32Logits, 4>, 160);
+    rc = logit_is_bf16 ? run(tv_flow_kernel<tvk::Bf16Logits, 4>, Shape<tvk::Bf16Logits, 4>::kThreads)
+                       : run(tv_flow_kernel<tvk::F32Logits, 4>, Shape<tvk::F32Logits, 4>::kThreads);
   if (rc) return rc;
   if (ev && cudaEventRecord(ev[3], stream) != cudaSuccess) return -5;
   return 0;
