@@ -3,9 +3,8 @@
 
 One step = one call of the library's verification (tv_verify_batch) over one
 batch of synthetic draft trees whose inputs are resident in HBM: the row
-normalisers of every internal row, the serial leaf-to-root traversal of
-every tree with its vocabulary-wide rejection passes, and the bonus-token
-draw.  L2 is flushed (a 256 MiB write) before every timed step, outside the
+normalisers the traversal needs, the serial leaf-to-root traversal of every
+tree with its vocabulary-wide rejection passes, and the bonus-token draw.  L2 is flushed (a 256 MiB write) before every timed step, outside the
 timed interval.  Times are CUDA-event device times on the launching stream.
 
 Prints ONE JSON line (rank 0).  ``--impl reference`` times the CPU oracle
@@ -164,20 +163,22 @@ def time_oracle(sample_dir, n_trees, temperature, pool, reps=1):
 
 # ---------------------------------------------------------- helpers ---------
 
-def algorithmic_bytes(parents, stats, V, logit_bytes):
-    """Per tree: one target row per internal node, one draft row per node with
-    at least one rejection pass, the accepted leaf's target row (the eager
-    reading of Algorithm 3's initialisation)."""
+def algorithmic_bytes(stats, tau, V, logit_bytes):
+    """Bytes of target logits and draft probabilities the verification has to
+    read, per tree: one target row for every normaliser computed (stats column
+    4), one target row and one draft row for every S-computation of
+    Eqs. (1)/(3) (column 1: each pass depends on the distribution the previous
+    one left), and one row (target only for an original leaf, target and draft
+    for a residual) for the bonus draw.  Returns (normaliser bytes, pass and
+    bonus bytes)."""
     import torch
-    B, R = parents.shape
-    has_child = torch.zeros(B, R, dtype=torch.bool, device=parents.device)
-    p = parents[:, 1:].long()
-    has_child.scatter_(1, p.clamp(min=0), True)
-    n_int = has_child.sum(1).to(torch.int64)
-    rej = stats[:, 2].to(torch.int64)
+    valid = tau >= 0
+    norm = stats[:, 4].to(torch.int64)
+    passes = stats[:, 1].to(torch.int64)
     leaf = stats[:, 3].to(torch.int64)
-    row_bytes = n_int * V * logit_bytes
-    other = rej * V * 4 + leaf * V * logit_bytes
+    row_bytes = norm * V * logit_bytes
+    bonus = torch.where(leaf > 0, V * logit_bytes, V * (logit_bytes + 4)) * valid.to(torch.int64)
+    other = passes * V * (logit_bytes + 4) + bonus
     return int(row_bytes.sum()), int(other.sum())
 
 
@@ -216,7 +217,7 @@ def main():
     _, tau_d, _, _, stats = v.verify(inp.parents, inp.tokens, inp.logits, inp.draft_probs,
                                      inp.temperature, inp.uniforms, debug=True)
     torch.cuda.synchronize(dev)
-    row_bytes, trav_bytes = algorithmic_bytes(inp.parents, stats, V, lb)
+    row_bytes, trav_bytes = algorithmic_bytes(stats, tau_d, V, lb)
     path_code, cluster, warps, stages = v.launch_shape(B, N)
     a_bytes = row_bytes + trav_bytes
     mean_tau1 = float(tau_d.float().mean()) + 1.0
@@ -337,7 +338,7 @@ def main():
         "data": "synthetic (seeded logits with Zipf rank prior, noisy-drafter probabilities, "
                 "EAGLE-shaped draft trees sampled without replacement)",
         "config": {"workload": w.name, "batch": B, "vocab": V, "nodes": N,
-                   "internal_rows": int(row_bytes // (V * lb) // B) if B else 0,
+                   "normalised_rows_per_tree": round(row_bytes / (V * lb) / B, 3) if B else 0,
                    "logit_dtype": "bf16" if lb == 2 else "fp32",
                    "temperature": w.temperature, "sigma": w.sigma, "seed": args.seed,
                    "l2": "flushed by a 256 MiB write before every timed step (untimed)",

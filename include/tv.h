@@ -152,10 +152,15 @@ int tv_verify_batch(tv_handle* h, int B, int N, const int32_t* parents,
  *               moment it was tested (Algorithm 3's eta < p test); 0 for a node
  *               removed because its rate reached 0 (§3.2); NaN for nodes never
  *               tested; entry 0 (root) NaN.
- *   out_stats   [B][4] int32 (device): { number of tests, number of
+ *   out_stats   [B][5] int32 (device): { number of tests, number of
  *               S-computations (Eqs. (1)/(3), one vocabulary pass each), number
  *               of distinct nodes with at least one S-computation, 1 if the
- *               bonus token came from an original leaf's row else 0 }.
+ *               bonus token came from an original leaf's row else 0, number of
+ *               target rows whose normaliser (softmax denominator) the call
+ *               computed }.  The first four follow from Algorithm 3; the last
+ *               depends on the kernel path (the three-kernel path normalises
+ *               every internal row, the single-kernel paths only the rows the
+ *               traversal reaches).
  * Either pointer may be NULL.  Other arguments and errors as tv_verify_batch.
  */
 int tv_verify_batch_debug(tv_handle* h, int B, int N, const int32_t* parents,

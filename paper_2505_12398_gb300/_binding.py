@@ -161,7 +161,7 @@ class Verifier:
         sp = _stream_ptr(stream)
         if debug:
             node_p = torch.empty(B, N + 1, dtype=torch.float32, device=self.device)
-            stats = torch.empty(B, 4, dtype=torch.int32, device=self.device)
+            stats = torch.empty(B, 5, dtype=torch.int32, device=self.device)
             rc = self.lib.tv_verify_batch_debug(
                 self.handle, B, N, _ptr(parents), _ptr(tokens), _ptr(logits), _ptr(drafts),
                 float(temperature), _ptr(uniforms), _ptr(path), _ptr(tau), _ptr(bonus),

@@ -24,7 +24,7 @@ struct tv_handle {
   int smem_per_sm = 0;
   int smem_per_block = 0;
   int force_ncw = 0, force_c = 0, force_stages = 0;   // tuning override (TV_FUSED_PLAN)
-  int flow_force[4] = {0, 0, 0, 0};                    // tuning override (TV_FLOW_PLAN)
+  int flow_force[5] = {0, 0, 0, 0, 0};                 // tuning override (TV_FLOW_PLAN)
   // device workspace
   int32_t* row_list = nullptr;   // [max_batch * (max_nodes + 1)]
   int32_t* n_rows = nullptr;     // [1]
@@ -52,13 +52,13 @@ enum Path { kPathThree = 0, kPathCluster = 1, kPathPersistent = 2 };
 
 FlowPlan flow_plan(const tv_handle* h, int R) {
   return tv_flow_plan(R, h->smem_per_sm, h->smem_per_block, h->flow_force[0], h->flow_force[1],
-                      h->flow_force[2], h->flow_force[3]);
+                      h->flow_force[2], h->flow_force[3], h->flow_force[4]);
 }
 
 // Smallest slice the persistent kernel may use on this handle (sizes its queue).
 int flow_min_slice(const tv_handle* h) {
   const FlowPlan p = flow_plan(h, h->max_nodes + 1);
-  return p.slice_pass < p.slice_stats ? p.slice_pass : p.slice_stats;
+  return p.slice_min;
 }
 
 Path choose_path(const tv_handle* h, int B, int R, FusedPlan* plan) {
@@ -202,11 +202,11 @@ int tv_create(tv_handle** out, int device, int vocab, int max_nodes, int max_bat
   // shape (tuning only; invalid values are ignored)
   if (const char* env = std::getenv("TV_FUSED_PLAN"))
     std::sscanf(env, "%d,%d,%d", &h->force_ncw, &h->force_c, &h->force_stages);
-  // TV_FLOW_PLAN="ncw,stages,slice_pass,slice_stats" does the same for the
-  // persistent kernel
+  // TV_FLOW_PLAN="ncw,stages,slice_pass,slice_stats,slice_min" does the same
+  // for the persistent kernel
   if (const char* env = std::getenv("TV_FLOW_PLAN"))
-    std::sscanf(env, "%d,%d,%d,%d", &h->flow_force[0], &h->flow_force[1], &h->flow_force[2],
-                &h->flow_force[3]);
+    std::sscanf(env, "%d,%d,%d,%d,%d", &h->flow_force[0], &h->flow_force[1], &h->flow_force[2],
+                &h->flow_force[3], &h->flow_force[4]);
   DeviceGuard guard(device);
   if (!guard.ok()) {
     delete h;
@@ -220,6 +220,14 @@ int tv_create(tv_handle** out, int device, int vocab, int max_nodes, int max_bat
             cudaMemset(h->status, 0, sizeof(uint32_t)) == cudaSuccess;
   if (ok && (vocab % 8) == 0 && !(flags & (TV_FLAG_UNFUSED | TV_FLAG_CLUSTER))) {
     // the queue's publication tags start at zero; calls use epochs 1, 2, ...
+    // the queue is sized for the smallest slice; for very large handles the
+    // smallest slice grows until the workspace stays within 1 GiB
+    const FlowPlan fp = flow_plan(h, max_nodes + 1);
+    int min_slice = fp.slice_min;
+    while (tv_flow_workspace_bytes(max_batch, max_nodes + 1, vocab, min_slice) > (1ull << 30) &&
+           min_slice < fp.slice_pass)
+      min_slice *= 2;
+    h->flow_force[4] = min_slice;
     h->flow_ws_bytes = tv_flow_workspace_bytes(max_batch, max_nodes + 1, vocab,
                                                flow_min_slice(h));
     ok = cudaMalloc(&h->flow_ws, h->flow_ws_bytes) == cudaSuccess &&

@@ -14,8 +14,10 @@
 // Each CTA is warp-specialised:
 //   * an owner warp runs the serial control of the CTA's current tree (tree
 //     set-up, combining partials, Eqs. (1)-(3), posting the next job);
-//   * a producer warp takes tickets, reads the queued slices and streams them
-//     into a shared-memory ring with 1-D bulk copies (TMA), one slice ahead;
+//   * a fetcher warp takes tickets and copies the queued slices into the
+//     CTA's slots, up to two slices ahead of the one being reduced;
+//   * a producer warp streams the fetched slices into a shared-memory ring
+//     with 1-D bulk copies (TMA);
 //   * NCW consumer warps reduce the ring stages and write each slice's
 //     partial result.
 // So the serial control of one tree overlaps the streaming of others, and
@@ -29,13 +31,15 @@
 //
 // Queue protocol: a poster reserves a range of slots with one atomicAdd on
 // the tail, writes the slots' bodies, fences, then stores each slot's tag
-// (call epoch, slot number).  A producer takes a ticket -- the next slot
+// (call epoch, slot number).  A fetcher takes a ticket -- the next slot
 // number, one atomicAdd on the head -- and processes that slot once its tag
 // appears.  Slots are never reused within a call; when the last tree is done
 // its owner writes an exit tag into every slot a ticket may still point to.
 // A slice's partial is one 64-bit store that doubles as its completion flag.
 #include <cuda_runtime.h>
 #include <stdint.h>
+
+#include <algorithm>
 
 #include "tv_control.cuh"
 #include "tv_device.cuh"
@@ -48,7 +52,7 @@ namespace flow {
 using namespace tvk::fused;
 
 constexpr int kMaxNCW = 8;
-constexpr int kSlots = 2;           // queued slices a CTA holds: one streaming, one ahead
+constexpr int kSlots = 3;           // queued slices a CTA holds: one streaming, two ahead
 constexpr int kPBuf = 256;          // partials of a job kept in shared memory by the poll
 constexpr unsigned long long kNoPart = ~0ull;   // a partial slot not written yet
 constexpr unsigned kNoTicket = 0xffffffffu;
@@ -61,6 +65,8 @@ enum : int {
   kNumCtr = 6
 };
 enum : int { kStageFirst = 1, kStageLast = 2, kStageExit = 4 };
+constexpr int kSlotExit = -1;       // ItemSlot::kind of the fetcher's "no more slices"
+constexpr int kItemNop = 6;         // FlowItem::kind of a reserved slot that carries no work
 
 // A queued slice as held by a CTA (the masks live in shared arrays of R).
 struct ItemSlot {
@@ -91,6 +97,12 @@ __device__ __forceinline__ unsigned ld_relaxed_u32(const unsigned* p) {
 __device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long long* p) {
   unsigned long long v;
   asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
   return v;
 }
 
@@ -128,7 +140,7 @@ __device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity) {
   return __all_sync(0xffffffffu, mbar_wait(bar, parity) ? 1 : 0) != 0;
 }
 
-// Sleep of an idle poller: 32 ns doubling to 256 ns; false once the wait has
+// Sleep of an idle poller: 32 ns, then 64 ns; false once the wait has
 // lasted kIdleNs (the caller aborts).
 struct Backoff {
   unsigned nap = 32u;
@@ -142,7 +154,7 @@ struct Backoff {
     if (since == 0ull) since = now;
     else if (now - since > kIdleNs) return false;
     __nanosleep(nap);
-    if (nap < 256u) nap <<= 1;
+    if (nap < 64u) nap <<= 1;
     return true;
   }
 };
@@ -152,7 +164,7 @@ struct Backoff {
 template <typename L, int kNCW>
 struct Shape {
   static constexpr int kConsumers = kNCW * 32;
-  static constexpr int kThreads = kConsumers + 64;   // + producer + owner warps
+  static constexpr int kThreads = kConsumers + 96;   // + producer, fetcher, owner warps
   static constexpr int kStageBytes = stage_bytes(kNCW);
   static constexpr int kSweep = kConsumers * kChunk;
   static constexpr int kLB = L::kBytes;
@@ -166,127 +178,161 @@ struct Smem {
   TreeSmem s;
   int* mtok;     // [kSlots][R] removed tokens of the held slices
   float* mval;   // [kSlots][R] their stored masses
+  float* u;      // [R + 1] the own tree's uniforms
   uint64_t* full_bar;
   uint64_t* empty_bar;
   uint64_t* slot_free;
+  uint64_t* slot_full;
   uint64_t* red_bar;
   Shared* sh;
 };
 
-// ------------------------------------------------------------ producer --
+// ------------------------------------------------------------- fetcher --
 
+// Takes tickets and copies the published slices into the CTA's slots, at most
+// kSlots - 1 ahead of the slice being reduced.
 template <typename L, int kNCW>
-__device__ void producer_role(const TravArgs& a, const FlowArgs& f, const Smem& m,
-                              int n_stages, int lane) {
-  using S = Shape<L, kNCW>;
-  using E = typename L::elem;
-  const int R = a.N + 1, V = a.V, B = a.B;
-  const E* logits = reinterpret_cast<const E*>(a.logits);
-  int stage = 0, phase = 0, slot = 0, slot_phase = 0;
-  unsigned ticket = kNoTicket, polls = 0u;
+__device__ void fetcher_role(const TravArgs& a, const FlowArgs& f, const Smem& m, int lane) {
+  const int R = a.N + 1, B = a.B;
+  int slot = 0, slot_phase = 0;
+  unsigned polls = 0u;
   Backoff wait;
-  bool aborted = false;
+  bool have_slot = false;
   for (;;) {
-    // ---- wait for the ticket's slot to be published (lane 0) ----
-    int cmd = 0;   // 0: keep polling, 1: a slice, 2: stop
-    if (lane == 0) {
-      if (ticket == kNoTicket) {
-        if (ld_relaxed_u32(&f.ctr[kCtrDone]) >= (unsigned)B) cmd = 2;   // nothing will come
-        else ticket = atomicAdd(&f.ctr[kCtrHead], 1u);
+    if (!have_slot) {
+      int ok = 1;
+      if (lane == 0) ok = mbar_wait(&m.slot_free[slot], slot_phase ^ 1) ? 1 : 0;
+      if (!__shfl_sync(0xffffffffu, ok, 0)) {
+        if (lane == 0) raise_abort(a, f);
+        return;   // the producer times out on its slot wait and stops the consumers
       }
-      if (cmd == 0) {
-        const unsigned long long want = (f.epoch << 32) | (unsigned long long)ticket;
+      have_slot = true;
+    }
+    ItemSlot& it = m.sh->slots[slot];
+    // ---- a ticket, then its slot's publication (lane 0) ----
+    int cmd = 0;   // 1: a slice, 2: stop, 3: a reserved slot without work
+    if (lane == 0) {
+      unsigned ticket = kNoTicket;
+      if (ld_relaxed_u32(&f.ctr[kCtrDone]) >= (unsigned)B) cmd = 2;   // nothing will come
+      else ticket = atomicAdd(&f.ctr[kCtrHead], 1u);
+      const unsigned long long want = (f.epoch << 32) | (unsigned long long)ticket;
+      while (cmd == 0) {
         const unsigned long long tag =
-            (ticket < (unsigned)f.cap) ? ld_relaxed_u64(&f.items[ticket].tag) : 0ull;
-        if ((++polls & 31u) == 0u && ld_relaxed_u32(&f.ctr[kCtrAbort])) {
-          cmd = 2;
-        } else if (tag == want) {
-          fence_gpu();
+            (ticket < (unsigned)f.cap) ? ld_acquire_u64(&f.items[ticket].tag) : 0ull;
+        if (tag == want) {
           cmd = 1;
-          wait.reset();
         } else if (tag == (want | kExitTag)) {
+          cmd = 2;
+        } else if ((++polls & 31u) == 0u && ld_relaxed_u32(&f.ctr[kCtrAbort])) {
           cmd = 2;
         } else if (!wait.idle()) {
           raise_abort(a, f);
           cmd = 2;
         }
       }
-    }
-    cmd = __shfl_sync(0xffffffffu, cmd, 0);
-    if (cmd == 2) break;
-    if (cmd == 0) continue;
-
-    // ---- copy the slice's description into a free slot ----
-    int ok = 1;
-    if (lane == 0) ok = mbar_wait(&m.slot_free[slot], slot_phase ^ 1) ? 1 : 0;
-    ok = __shfl_sync(0xffffffffu, ok, 0);
-    if (!ok) {
-      if (lane == 0) raise_abort(a, f);
-      aborted = true;
-      break;
-    }
-    ItemSlot& it = m.sh->slots[slot];
-    int b = 0, nmask = 0;
-    if (lane == 0) {
-      const int4* bp = reinterpret_cast<const int4*>(f.items + ticket);
-      const int4 w0 = __ldcg(bp), w1 = __ldcg(bp + 1), w2 = __ldcg(bp + 2);
-      it.b = w0.x; it.node = w0.y; it.row = w0.z; it.slice = w0.w;
-      it.kind = w1.x; it.slice_len = w1.y; it.nmask = w1.z;
-      it.alpha1 = __int_as_float(w2.x); it.beta = __int_as_float(w2.y);
-      it.rowmax = __int_as_float(w2.z);
-      b = w0.x;
-      nmask = w1.z;
-      ticket = kNoTicket;
-    }
-    b = __shfl_sync(0xffffffffu, b, 0);
-    nmask = __shfl_sync(0xffffffffu, nmask, 0);
-    for (int q = lane; q < nmask; q += 32) {
-      m.mtok[slot * R + q] = __ldcg(f.job_mtok + (size_t)b * R + q);
-      m.mval[slot * R + q] = __ldcg(f.job_mval + (size_t)b * R + q);
-    }
-    __syncwarp();
-
-    // ---- stream it through the ring ----
-    if (lane == 0) {
-      const bool pair = (it.kind == kJobPass || it.kind == kJobBonusRes);
-      const int per = pair ? S::kPairElems : S::kRowElems;
-      const int x0 = it.slice * it.slice_len;
-      const int x1 = min(V, x0 + it.slice_len);
-      const size_t row = ((size_t)b * R + it.node) * (size_t)V;
-      for (int x = x0; x < x1; x += per) {
-        const int n = min(per, x1 - x);
-        if (!mbar_wait(&m.empty_bar[stage], phase ^ 1)) {
-          raise_abort(a, f);
-          aborted = true;
-          break;
-        }
-        m.sh->meta[stage] = StageMeta{slot, x, n, (x == x0 ? kStageFirst : 0) |
-                                                      (x + n >= x1 ? kStageLast : 0)};
-        char* dst = m.ring + (size_t)stage * S::kStageBytes;
-        const uint32_t lbytes = (uint32_t)n * S::kLB;
-        const uint32_t qbytes = pair ? (uint32_t)n * 4u : 0u;
-        mbar_arrive_expect_tx(&m.full_bar[stage], lbytes + qbytes);
-        tma_load_1d(dst, logits + row + x, lbytes, &m.full_bar[stage]);
-        if (pair)
-          tma_load_1d(dst + (size_t)S::kPairElems * S::kLB, a.draft_probs + row + x, qbytes,
-                      &m.full_bar[stage]);
-        if (++stage == n_stages) { stage = 0; phase ^= 1; }
+      wait.reset();
+      int4 w[7];
+      if (cmd == 1) {
+        const int4* bp = reinterpret_cast<const int4*>(f.items + ticket);
+#pragma unroll
+        for (int k = 0; k < 7; ++k) w[k] = __ldcg(bp + k);   // one 112-byte read
+        if (w[1].x == kItemNop) cmd = 3;
+      }
+      if (cmd == 1) {
+        it.b = w[0].x; it.node = w[0].y; it.row = w[0].z; it.slice = w[0].w;
+        it.kind = w[1].x; it.slice_len = w[1].y; it.nmask = w[1].z;
+        it.alpha1 = __int_as_float(w[2].x); it.beta = __int_as_float(w[2].y);
+        it.rowmax = __int_as_float(w[2].z);
+        int* mt = m.mtok + slot * R;
+        float* mv = m.mval + slot * R;
+        const int ni = min(w[1].z, kFlowInlineMask);
+        const int tk[8] = {w[3].x, w[3].y, w[3].z, w[3].w, w[4].x, w[4].y, w[4].z, w[4].w};
+        const int vk[8] = {w[5].x, w[5].y, w[5].z, w[5].w, w[6].x, w[6].y, w[6].z, w[6].w};
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          if (q < ni) { mt[q] = tk[q]; mv[q] = __int_as_float(vk[q]); }
+      } else if (cmd == 2) {
+        it.kind = kSlotExit;
       }
     }
-    stage = __shfl_sync(0xffffffffu, stage, 0);
-    phase = __shfl_sync(0xffffffffu, phase, 0);
-    if (__shfl_sync(0xffffffffu, aborted ? 1 : 0, 0)) break;
+    cmd = __shfl_sync(0xffffffffu, cmd, 0);
+    __syncwarp();
+    if (cmd == 3) continue;   // keep the slot for the next ticket
+    if (cmd == 1) {
+      const int nmask = it.nmask;
+      if (nmask > kFlowInlineMask) {   // rare: the rest of a long mask list
+        const int b = it.b;
+        fence_gpu();
+        for (int q = kFlowInlineMask + lane; q < nmask; q += 32) {
+          m.mtok[slot * R + q] = __ldcg(f.job_mtok + (size_t)b * R + q);
+          m.mval[slot * R + q] = __ldcg(f.job_mval + (size_t)b * R + q);
+        }
+      }
+      __syncwarp();
+    }
+    if (lane == 0) mbar_arrive(&m.slot_full[slot]);   // release: the slot's contents
+    if (cmd == 2) return;
+    have_slot = false;
+    if (++slot == kSlots) { slot = 0; slot_phase ^= 1; }
+  }
+}
+
+// ------------------------------------------------------------ producer --
+
+// Streams the fetched slices through the ring, in slot order (one lane).
+template <typename L, int kNCW>
+__device__ void producer_loop(const TravArgs& a, const FlowArgs& f, const Smem& m,
+                              int n_stages) {
+  using S = Shape<L, kNCW>;
+  using E = typename L::elem;
+  const int R = a.N + 1, V = a.V;
+  const E* logits = reinterpret_cast<const E*>(a.logits);
+  int stage = 0, phase = 0, slot = 0, slot_phase = 0;
+  for (;;) {
+    if (!mbar_wait(&m.slot_full[slot], slot_phase)) {
+      raise_abort(a, f);
+      return;   // the consumers time out on their stage wait
+    }
+    const ItemSlot& it = m.sh->slots[slot];
+    if (it.kind == kSlotExit) break;
+    const bool pair = (it.kind == kJobPass || it.kind == kJobBonusRes);
+    const int per = pair ? S::kPairElems : S::kRowElems;
+    const int x0 = it.slice * it.slice_len;
+    const int x1 = min(V, x0 + it.slice_len);
+    const size_t row = ((size_t)it.b * R + it.node) * (size_t)V;
+    for (int x = x0; x < x1; x += per) {
+      const int n = min(per, x1 - x);
+      if (!mbar_wait(&m.empty_bar[stage], phase ^ 1)) {
+        raise_abort(a, f);
+        return;
+      }
+      m.sh->meta[stage] = StageMeta{slot, x, n, (x == x0 ? kStageFirst : 0) |
+                                                    (x + n >= x1 ? kStageLast : 0)};
+      char* dst = m.ring + (size_t)stage * S::kStageBytes;
+      const uint32_t lbytes = (uint32_t)n * S::kLB;
+      const uint32_t qbytes = pair ? (uint32_t)n * 4u : 0u;
+      mbar_arrive_expect_tx(&m.full_bar[stage], lbytes + qbytes);
+      tma_load_1d(dst, logits + row + x, lbytes, &m.full_bar[stage]);
+      if (pair)
+        tma_load_1d(dst + (size_t)S::kPairElems * S::kLB, a.draft_probs + row + x, qbytes,
+                    &m.full_bar[stage]);
+      if (++stage == n_stages) { stage = 0; phase ^= 1; }
+    }
     if (++slot == kSlots) { slot = 0; slot_phase ^= 1; }
   }
   // ---- tell the consumers to stop ----
-  if (lane == 0 && !aborted) {
-    if (mbar_wait(&m.empty_bar[stage], phase ^ 1)) {
-      m.sh->meta[stage] = StageMeta{0, 0, 0, kStageExit};
-      mbar_arrive(&m.full_bar[stage]);
-    } else {
-      raise_abort(a, f);
-    }
+  if (mbar_wait(&m.empty_bar[stage], phase ^ 1)) {
+    m.sh->meta[stage] = StageMeta{0, 0, 0, kStageExit};
+    mbar_arrive(&m.full_bar[stage]);
+  } else {
+    raise_abort(a, f);
   }
+}
+
+template <typename L, int kNCW>
+__device__ void producer_role(const TravArgs& a, const FlowArgs& f, const Smem& m,
+                              int n_stages, int lane) {
+  if (lane == 0) producer_loop<L, kNCW>(a, f, m, n_stages);
   __syncwarp();
 }
 
@@ -522,18 +568,67 @@ __device__ void consumer_role(const TravArgs& a, const FlowArgs& f, const Smem& 
 
 // --------------------------------------------------------------- owner --
 
-// Publishes the own tree's current job (ctl.job) as slice items.
+// Queue slots reserved ahead of the job that will use them (see owner_role).
+struct Reserve {
+  unsigned base;
+  int n;       // 0: none
+  int slice;
+};
+
+// Tokens per slice: enough slices per row to give every CTA one when each
+// remaining tree has a job out, between the plan's largest and smallest
+// slice.  Early on (many trees) this keeps slices large; towards the end,
+// when a few trees' chains of jobs set the time, their jobs spread over more
+// CTAs.  `done` is the number of finished trees as last read.
+__device__ __forceinline__ int adaptive_slice(const FlowArgs& f, int V, int B, bool stats,
+                                              int n_rows, unsigned done) {
+  const int largest = stats ? f.slice_stats : f.slice_pass;
+  const int active = max(1, B - (int)done);
+  const int per_row = max(1, (int)gridDim.x / (active * n_rows));
+  int want = (V + per_row - 1) / per_row;
+  want = (want + kTileElems - 1) / kTileElems * kTileElems;
+  return max(f.slice_min, min(largest, want));
+}
+
+// Writes "no work" items into reserved slots [base, base + n) (before the
+// caller's fence) ...
+__device__ __forceinline__ void nop_bodies(const FlowArgs& f, unsigned base, int n, int lane) {
+  for (int q = lane; q < n; q += 32)
+    __stcg(reinterpret_cast<int4*>(f.items + base + q) + 1, make_int4(kItemNop, 0, 0, 0));
+}
+
+// ... and, after it, their tags.
+__device__ __forceinline__ void nop_tags(const FlowArgs& f, unsigned base, int n, int lane) {
+  for (int q = lane; q < n; q += 32)
+    st_relaxed_u64(&f.items[base + q].tag, (f.epoch << 32) | (unsigned long long)(base + q));
+}
+
+// Publishes reserved slots that no job will use.
+__device__ void post_nops(const TravArgs& a, const FlowArgs& f, Reserve spec, int lane) {
+  if ((size_t)spec.base + spec.n + kMaxGrid > (size_t)f.cap) {
+    if (lane == 0) raise_abort(a, f);
+    return;
+  }
+  nop_bodies(f, spec.base, spec.n, lane);
+  fence_gpu();
+  __syncwarp();
+  nop_tags(f, spec.base, spec.n, lane);
+}
+
+// Publishes the own tree's current job (ctl.job) as slice items.  A pass may
+// use the slots reserved in `spec`; otherwise those become "no work" items.
 __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const FlowArgs& f,
-                         int b, int V, int lane) {
+                         int b, int V, int lane, unsigned done, Reserve spec) {
   const Job& j = sh.ctl.job;
   const bool stats = (j.kind == kJobStats);
   const int n_rows = stats ? j.n_rows : 1;
-  const int slice = stats ? f.slice_stats : f.slice_pass;
+  const bool use_spec = spec.n > 0 && j.kind == kJobPass;
+  const int slice = use_spec ? spec.slice : adaptive_slice(f, V, a.B, stats, n_rows, done);
   const int K = (V + slice - 1) / slice;
   const int nmask = (j.kind == kJobPass || j.kind == kJobBonusRes) ? j.nmask : 0;
   const int n = n_rows * K;
   const size_t R = (size_t)f.R;
-  for (int q = lane; q < nmask; q += 32) {
+  for (int q = kFlowInlineMask + lane; q < nmask; q += 32) {   // beyond the inline ones
     f.job_mtok[b * R + q] = s.mask_tok[q];
     f.job_mval[b * R + q] = s.mask_val[q];
   }
@@ -542,29 +637,53 @@ __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const
     const int r = q / K;
     __stcg(f.part + ((size_t)b * R + r) * f.Kmax + (q - r * K), kNoPart);
   }
-  unsigned base = 0u;
-  if (lane == 0) base = atomicAdd(&f.ctr[kCtrTail], (unsigned)n);
-  base = __shfl_sync(0xffffffffu, base, 0);
+  unsigned base = spec.base;
+  if (!use_spec) {
+    if (lane == 0) base = atomicAdd(&f.ctr[kCtrTail], (unsigned)n);
+    base = __shfl_sync(0xffffffffu, base, 0);
+  }
   // the last kMaxGrid slots are kept for exit tags; a correctly sized queue
   // never reaches them
-  if ((size_t)base + n + kMaxGrid > (size_t)f.cap) {
+  if ((size_t)base + n + kMaxGrid > (size_t)f.cap ||
+      (spec.n > 0 && (size_t)spec.base + spec.n + kMaxGrid > (size_t)f.cap)) {
     if (lane == 0) raise_abort(a, f);
     return;
   }
+  if (spec.n > 0 && !use_spec) nop_bodies(f, spec.base, spec.n, lane);
   const int4 w1 = make_int4(j.kind, slice, nmask, 0);
   const int4 w2 = make_int4(__float_as_int(j.alpha1), __float_as_int(j.beta),
                             __float_as_int(j.rowmax), 0);
+  int tk[kFlowInlineMask];
+  float vk[kFlowInlineMask];
+#pragma unroll
+  for (int q = 0; q < kFlowInlineMask; ++q) {
+    tk[q] = (q < nmask) ? s.mask_tok[q] : 0x7fffffff;
+    vk[q] = (q < nmask) ? s.mask_val[q] : 0.f;
+  }
+  const int4 w3 = make_int4(tk[0], tk[1], tk[2], tk[3]);
+  const int4 w4 = make_int4(tk[4], tk[5], tk[6], tk[7]);
+  const int4 w5 = make_int4(__float_as_int(vk[0]), __float_as_int(vk[1]),
+                            __float_as_int(vk[2]), __float_as_int(vk[3]));
+  const int4 w6 = make_int4(__float_as_int(vk[4]), __float_as_int(vk[5]),
+                            __float_as_int(vk[6]), __float_as_int(vk[7]));
   for (int q = lane; q < n; q += 32) {
     const int r = q / K;
     int4* w = reinterpret_cast<int4*>(f.items + base + q);
     __stcg(w, make_int4(b, stats ? s.job_rows[r] : j.node, r, q - r * K));
     __stcg(w + 1, w1);
     __stcg(w + 2, w2);
+    if (nmask > 0) {
+      __stcg(w + 3, w3);
+      __stcg(w + 4, w4);
+      __stcg(w + 5, w5);
+      __stcg(w + 6, w6);
+    }
   }
   fence_gpu();   // bodies, masks and partial resets before tags
   __syncwarp();
   for (int q = lane; q < n; q += 32)
     st_relaxed_u64(&f.items[base + q].tag, (f.epoch << 32) | (unsigned long long)(base + q));
+  if (spec.n > 0 && !use_spec) nop_tags(f, spec.base, spec.n, lane);
   if (lane == 0) {
     sh.outstanding = n;
     sh.jkind = j.kind;
@@ -576,8 +695,8 @@ __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const
 
 // Structure, validation and gathers of tree b; leaves ctl ready to run.
 template <typename L>
-__device__ void owner_new_tree(const TravArgs& a, const TreeSmem& s, Shared& sh, int b,
-                               int lane) {
+__device__ void owner_new_tree(const TravArgs& a, const TreeSmem& s, Shared& sh, float* u,
+                               int b, int lane) {
   const int R = a.N + 1, V = a.V;
   const size_t row0 = (size_t)b * R;
   const typename L::elem* logits = reinterpret_cast<const typename L::elem*>(a.logits);
@@ -592,6 +711,7 @@ __device__ void owner_new_tree(const TravArgs& a, const TreeSmem& s, Shared& sh,
     c.n_tests = c.n_passes = 0;
     c.job.kind = 0;
   }
+  for (int i = lane; i <= R; i += 32) u[i] = a.uniforms[row0 + b + i];
   for (int i = lane; i < R; i += 32) {
     s.par[i] = a.parents[row0 + i];
     s.tok[i] = a.tokens[row0 + i];
@@ -649,7 +769,7 @@ __device__ void owner_new_tree(const TravArgs& a, const TreeSmem& s, Shared& sh,
     sh.ctl.bad = bad;
     if (bad == 0u) {
       s.p[0] = 1.0;
-      control_step(s, sh.ctl, a.uniforms + row0 + b);
+      control_step(s, sh.ctl, u);
     } else {
       sh.ctl.job.kind = kJobDone;
     }
@@ -660,7 +780,7 @@ __device__ void owner_new_tree(const TravArgs& a, const TreeSmem& s, Shared& sh,
 // Combines the finished job's partials (sh.pbuf or global) and advances.
 template <typename L>
 __device__ void owner_combine(const TravArgs& a, const FlowArgs& f, const TreeSmem& s,
-                              Shared& sh, int b, int lane) {
+                              Shared& sh, const float* u, int b, int lane) {
   const int R = a.N + 1, V = a.V;
   const size_t row0 = (size_t)b * R;
   const float c_hi = a.c_hi, c_lo = a.c_lo;
@@ -672,28 +792,33 @@ __device__ void owner_combine(const TravArgs& a, const FlowArgs& f, const TreeSm
                    : unpack_part(__ldcg(f.part + (row0 + r) * f.Kmax + k));
   };
   if (sh.jkind == kJobStats) {
-    // normaliser of each row from its slices, then its children's M_b0
-    for (int r = 0; r < sh.jrows; ++r) {
+    // the rows' normalisers from their slices, one lane per row ...
+    bool bad_row = false;
+    for (int r = lane; r < sh.jrows; r += 32) {
       float M = TV_NEG_INF;
-      for (int k2 = lane; k2 < K; k2 += 32) M = fmaxf(M, part_of(r, k2).x);
-      M = warp_max(M);
+      for (int k2 = 0; k2 < K; ++k2) M = fmaxf(M, part_of(r, k2).x);
       float S = 0.f;
-      for (int k2 = lane; k2 < K; k2 += 32) {
+      for (int k2 = 0; k2 < K; ++k2) {
         const float2 pk = part_of(r, k2);
         if (pk.x != TV_NEG_INF) S += pk.y * L::exp_rel(pk.x, M, c_hi, c_lo);
       }
-      S = warp_sum(S);
       const int node = s.job_rows[r];
-      if (lane == 0) {
-        s.rowm[node] = M;
-        s.rows[node] = S;
-        s.invs[node] = 1.0 / (double)S;
-        if (!(S > 0.f)) sh.ctl.bad |= 64u;
-      }
-      __syncwarp();
-      children_mb0(s, node, a.c, lane);
-      __syncwarp();
+      s.rowm[node] = M;
+      s.rows[node] = S;
+      s.invs[node] = 1.0 / (double)S;
+      bad_row |= !(S > 0.f);
     }
+    if (__any_sync(0xffffffffu, bad_row) && lane == 0) sh.ctl.bad |= 64u;
+    __syncwarp();
+    // ... then M_b^(0) of those rows' children, one lane per node (the same
+    // value children_mb0 gives, see there)
+    for (int i = lane + 1; i < R; i += 32) {
+      const int p = s.par[i];
+      bool mine = false;
+      for (int r = 0; r < sh.jrows; ++r) mine |= (s.job_rows[r] == p);
+      if (mine) s.mb0[i] = exp2(((double)s.gl[i] - (double)s.rowm[p]) * a.c) * s.invs[p];
+    }
+    __syncwarp();
   } else if (sh.jkind == kJobPass) {
     float S = 0.f;
     for (int k2 = lane; k2 < K; k2 += 32) S += part_of(0, k2).x;
@@ -719,7 +844,7 @@ __device__ void owner_combine(const TravArgs& a, const FlowArgs& f, const TreeSm
       W += pk.y * slice_scale(pk.x);
     }
     W = warp_sum(W);
-    const float target = a.uniforms[row0 + b + R] * W;
+    const float target = u[R] * W;
     // first slice whose running total exceeds the target (warp scan per 32 slices)
     int owner = -1, last_pos = -1;
     float before = 0.f, scale = 0.f, last_before = 0.f, last_scale = 0.f, base = 0.f;
@@ -863,7 +988,7 @@ __device__ void owner_combine(const TravArgs& a, const FlowArgs& f, const TreeSm
   __syncwarp();
   if (lane == 0 && sh.ctl.job.kind != kJobDone) {
     if (sh.ctl.bad & 64u) sh.ctl.job.kind = kJobDone;
-    else control_step(s, sh.ctl, a.uniforms + row0 + b);
+    else control_step(s, sh.ctl, u);
   }
   __syncwarp();
 }
@@ -895,11 +1020,14 @@ __device__ bool owner_finish(const TravArgs& a, const FlowArgs& f, const TreeSme
     if (a.out_stats) {
       int distinct = 0;
       for (int i = 0; i < R; ++i) distinct += (s.npass[i] > 0);
-      int32_t* o = a.out_stats + (size_t)b * 4;
+      int normalised = 0;
+      for (int i = 0; i < R; ++i) normalised += (s.rows[i] > 0.f);
+      int32_t* o = a.out_stats + (size_t)b * 5;
       o[0] = ok ? sh.ctl.n_tests : 0;
       o[1] = ok ? sh.ctl.n_passes : 0;
       o[2] = ok ? distinct : 0;
       o[3] = (acc_node >= 0 && s.first[acc_node] < 0) ? 1 : 0;
+      o[4] = ok ? normalised : 0;
     }
     if (sh.ctl.bad) atomicOr(a.status, sh.ctl.bad);
     f.finished[b] = (unsigned)f.epoch;
@@ -918,6 +1046,8 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
   int my_tree = -1;
   unsigned polls = 0u;
   Backoff wait;
+  unsigned done_est = 0u;      // trees finished, as read after the last post
+  Reserve spec{0u, 0, 0};      // slots reserved for the next job (lane 0's copy counts)
   for (;;) {
     __syncwarp();   // lane 0's updates of sh (job shape, control state) seen by all lanes
     if (my_tree < 0) {
@@ -928,7 +1058,7 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
       t = __shfl_sync(0xffffffffu, t, 0);
       if (t >= (unsigned)B) break;   // no trees left for this CTA to own
       my_tree = (int)t;
-      owner_new_tree<L>(a, s, sh, my_tree, lane);
+      owner_new_tree<L>(a, s, sh, m.u, my_tree, lane);
     } else {
       // poll the own job's partials (kept in pbuf for the combine)
       const int nout = sh.outstanding;
@@ -955,12 +1085,25 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
         continue;
       }
       wait.reset();
+      // after a pass the next job is most often a pass of the same row size:
+      // reserve its queue slots now, so that the reservation's round trip
+      // overlaps the combine and the control step
+      if (lane == 0 && sh.jkind == kJobPass) {
+        spec.slice = adaptive_slice(f, V, B, false, 1, done_est);
+        spec.n = (V + spec.slice - 1) / spec.slice;
+        spec.base = atomicAdd(&f.ctr[kCtrTail], (unsigned)spec.n);
+      }
       // the bonus draw reads tiles written before its partials
       if (sh.jkind == kJobBonusLeaf || sh.jkind == kJobBonusRes) fence_gpu();
       __syncwarp();
-      owner_combine<L>(a, f, s, sh, my_tree, lane);
+      owner_combine<L>(a, f, s, sh, m.u, my_tree, lane);
     }
+    spec.base = __shfl_sync(0xffffffffu, spec.base, 0);
+    spec.n = __shfl_sync(0xffffffffu, spec.n, 0);
+    spec.slice = __shfl_sync(0xffffffffu, spec.slice, 0);
     if (sh.ctl.job.kind == kJobDone) {
+      if (spec.n > 0) post_nops(a, f, spec, lane);   // before the tree counts as done
+      spec.n = 0;
       const bool last = owner_finish(a, f, s, sh, my_tree, lane);
       my_tree = -1;
       if (last) {
@@ -978,7 +1121,9 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
           st_relaxed_u64(&f.items[q].tag, (f.epoch << 32) | q | kExitTag);
       }
     } else {
-      post_job(s, sh, a, f, my_tree, V, lane);
+      post_job(s, sh, a, f, my_tree, V, lane, __shfl_sync(0xffffffffu, done_est, 0), spec);
+      spec.n = 0;
+      if (lane == 0) done_est = ld_relaxed_u32(&f.ctr[kCtrDone]);   // used at the next job
     }
   }
 }
@@ -994,6 +1139,7 @@ __global__ void __launch_bounds__(Shape<L, kNCW>::kThreads, 16 / kNCW)
   __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
   __shared__ __align__(8) uint64_t red_bar[kMaxStages];
   __shared__ __align__(8) uint64_t slot_free[kSlots];
+  __shared__ __align__(8) uint64_t slot_full[kSlots];
   __shared__ Shared sh;
 
   const int R = args.N + 1;
@@ -1004,9 +1150,11 @@ __global__ void __launch_bounds__(Shape<L, kNCW>::kThreads, 16 / kNCW)
   m.s = carve_tree_nt(tree_base, R, 0);
   m.mtok = reinterpret_cast<int*>(tree_base + ((tree_smem_bytes_nt(R, 0) + 15) & ~(size_t)15));
   m.mval = reinterpret_cast<float*>(m.mtok + kSlots * R);
+  m.u = m.mval + kSlots * R;
   m.full_bar = full_bar;
   m.empty_bar = empty_bar;
   m.slot_free = slot_free;
+  m.slot_full = slot_full;
   m.red_bar = red_bar;
   m.sh = &sh;
 
@@ -1016,7 +1164,10 @@ __global__ void __launch_bounds__(Shape<L, kNCW>::kThreads, 16 / kNCW)
       mbar_init(&empty_bar[k], kNCW);
       mbar_init(&red_bar[k], kNCW);
     }
-    for (int k = 0; k < kSlots; ++k) mbar_init(&slot_free[k], kNCW);
+    for (int k = 0; k < kSlots; ++k) {
+      mbar_init(&slot_free[k], kNCW);
+      mbar_init(&slot_full[k], 1);
+    }
     fence_mbar_init();
     sh.outstanding = 0;
   }
@@ -1024,6 +1175,7 @@ __global__ void __launch_bounds__(Shape<L, kNCW>::kThreads, 16 / kNCW)
 
   if (wid < kNCW) consumer_role<L, kNCW>(args, f, m, n_stages, wid, lane);
   else if (wid == kNCW) producer_role<L, kNCW>(args, f, m, n_stages, lane);
+  else if (wid == kNCW + 1) fetcher_role<L, kNCW>(args, f, m, lane);
   else owner_role<L>(args, f, m, lane);
 
   // ---------------- exit ----------------
@@ -1061,8 +1213,9 @@ FlowLayout flow_layout(int B, int R, int V, int min_slice) {
   FlowLayout l;
   l.kmax = (size_t)((V + min_slice - 1) / min_slice);
   // per tree: at most R rows normalised and at most R - 1 passes plus the
-  // bonus draw, each at most kmax slices; then room for the exit tags
-  l.cap = (size_t)B * (2 * (size_t)R + 1) * l.kmax + tvk::flow::kMaxGrid;
+  // bonus draw, each at most kmax slices, and for each job at most one range
+  // reserved ahead and left unused; then room for the exit tags
+  l.cap = (size_t)B * (4 * (size_t)R + 2) * l.kmax + tvk::flow::kMaxGrid;
   l.ntiles = (size_t)((V + tvk::fused::kTileElems - 1) / tvk::fused::kTileElems);
   return l;
 }
@@ -1072,7 +1225,7 @@ size_t up256(size_t n) { return (n + 255) & ~static_cast<size_t>(255); }
 size_t flow_smem_bytes(int R, int ncw, int stages) {
   return (size_t)stages * tvk::fused::stage_bytes(ncw) +
          ((tvk::fused::tree_smem_bytes_nt(R, 0) + 15) & ~(size_t)15) +
-         (size_t)tvk::flow::kSlots * R * 8 + 64;
+         (size_t)tvk::flow::kSlots * R * 8 + (size_t)(R + 1) * 4 + 64;
 }
 
 }  // namespace
@@ -1086,8 +1239,7 @@ size_t tv_flow_workspace_bytes(int B, int R, int V, int min_slice) {
 
 int tv_flow_bind(void* base, size_t bytes, int B, int R, int V, const FlowPlan& plan,
                  FlowArgs* f) {
-  const FlowLayout l = flow_layout(B, R, V, plan.slice_pass < plan.slice_stats
-                                                ? plan.slice_pass : plan.slice_stats);
+  const FlowLayout l = flow_layout(B, R, V, plan.slice_min);
   char* p = static_cast<char*>(base);
   auto take = [&](size_t n) {
     char* q = p;
@@ -1107,15 +1259,19 @@ int tv_flow_bind(void* base, size_t bytes, int B, int R, int V, const FlowPlan& 
   f->ntiles = (int)l.ntiles;
   f->slice_pass = plan.slice_pass;
   f->slice_stats = plan.slice_stats;
+  f->slice_min = plan.slice_min;
   return (size_t)(p - static_cast<char*>(base)) <= bytes ? 0 : -4;
 }
 
 FlowPlan tv_flow_plan(int R, int smem_per_sm, int smem_per_block, int force_ncw,
-                      int force_stages, int force_slice_pass, int force_slice_stats) {
+                      int force_stages, int force_slice_pass, int force_slice_stats,
+                      int force_slice_min) {
   FlowPlan p;
   if (force_ncw == 4 || force_ncw == 8) p.ncw = force_ncw;
   if (force_slice_pass >= 256 && force_slice_pass % 256 == 0) p.slice_pass = force_slice_pass;
   if (force_slice_stats >= 256 && force_slice_stats % 256 == 0) p.slice_stats = force_slice_stats;
+  if (force_slice_min >= 256 && force_slice_min % 256 == 0) p.slice_min = force_slice_min;
+  p.slice_min = std::min(p.slice_min, std::min(p.slice_pass, p.slice_stats));
   const int per_sm = 16 / p.ncw;   // CTAs per SM the kernel is built for
   if (force_stages >= 2 && force_stages <= tvk::fused::kMaxStages) {
     p.stages = force_stages;

@@ -728,11 +728,14 @@ __global__ void __launch_bounds__(kTravThreads, 1) tv_traverse_kernel(TravArgs a
     if (args.out_stats) {
       int distinct = 0;
       for (int i = 0; i < R; ++i) distinct += (s.npass[i] > 0);
-      int32_t* o = args.out_stats + (size_t)b * 4;
+      int internal = 0;
+      for (int i = 0; i < R; ++i) internal += (s.first[i] >= 0);
+      int32_t* o = args.out_stats + (size_t)b * 5;
       o[0] = ok ? st.n_tests : 0;
       o[1] = ok ? st.n_passes : 0;
       o[2] = ok ? distinct : 0;
       o[3] = (acc_node >= 0 && s.first[acc_node] < 0) ? 1 : 0;
+      o[4] = ok ? internal : 0;
     }
     if (ctl.bad) atomicOr(args.status, ctl.bad);
   }

@@ -53,11 +53,15 @@ int tv_launch_all(const TravArgs& a, int logit_is_bf16, int* row_list, int* n_ro
 // ---- persistent load-balanced kernel (tv_flow.cu) ----
 
 // One slot of the persistent kernel's work queue: a slice of one tree's
-// current vocabulary job, self-contained so that a claim is one 48-byte read.
-struct __align__(64) FlowItem {
+// current vocabulary job, self-contained (with up to kFlowInlineMask removed
+// tokens) so that a claim is one 128-byte read.
+constexpr int kFlowInlineMask = 8;
+struct __align__(128) FlowItem {
   int tree, node, row, slice;   // tree, target row, row index within the job, slice
   int kind, slice_len, nmask, pad0;
   float alpha1, beta, rowmax, pad1;
+  int mtok[kFlowInlineMask];    // first removed tokens of the row (ascending)
+  float mval[kFlowInlineMask];  // their stored masses
   unsigned long long tag;       // epoch << 32 | slot, stored after the rest
   unsigned long long pad2;
 };
@@ -75,22 +79,25 @@ struct FlowArgs {
   float2* tiles;                 // [B][ntiles] per-tile sums of the bonus draw
   unsigned long long epoch;      // differs between calls sharing the workspace
   int cap, R, Kmax, ntiles;
-  int slice_pass, slice_stats;   // tokens per slice (multiples of 256)
+  int slice_pass, slice_stats;   // largest tokens per slice (multiples of 256)
+  int slice_min;                 // smallest tokens per slice (multiple of 256)
 };
 
 // Launch shape of the persistent kernel.
 struct FlowPlan {
   int ncw = 4;                   // consumer warps per CTA (4 or 8)
   int stages = 3;                // ring stages of 3 KB per consumer warp
-  int slice_pass = 8192;         // tokens per slice of a pass / bonus draw
-  int slice_stats = 16384;       // tokens per slice of a row normaliser
+  int slice_pass = 8192;         // largest slice of a pass / bonus draw (tokens)
+  int slice_stats = 16384;       // largest slice of a row normaliser (tokens)
+  int slice_min = 2048;          // slices shrink to this as fewer trees remain
   size_t smem = 0;
   bool ok = false;
 };
 
 // Default plan for R = N+1 rows (tuning overrides: force_* > 0).
 FlowPlan tv_flow_plan(int R, int smem_per_sm, int smem_per_block, int force_ncw,
-                      int force_stages, int force_slice_pass, int force_slice_stats);
+                      int force_stages, int force_slice_pass, int force_slice_stats,
+                      int force_slice_min);
 // Workspace for slices of at least `min_slice` tokens.
 size_t tv_flow_workspace_bytes(int B, int R, int V, int min_slice);
 // Carves the workspace; 0 on success, TV_ERR_CAPACITY if `bytes` is too small.

@@ -644,11 +644,14 @@ __global__ void __launch_bounds__(NCW * 32 + 32, 16 / NCW) tv_tree_kernel(TravAr
         if (args.out_stats) {
           int distinct = 0;
           for (int i = 0; i < R; ++i) distinct += (s.npass[i] > 0);
-          int32_t* o = args.out_stats + (size_t)b * 4;
+          int normalised = 0;
+          for (int i = 0; i < R; ++i) normalised += (s.rows[i] > 0.f);
+          int32_t* o = args.out_stats + (size_t)b * 5;
           o[0] = ok ? ctl.n_tests : 0;
           o[1] = ok ? ctl.n_passes : 0;
           o[2] = ok ? distinct : 0;
           o[3] = (acc_node >= 0 && s.first[acc_node] < 0) ? 1 : 0;
+          o[4] = ok ? normalised : 0;
         }
         if (ctl.bad) atomicOr(args.status, ctl.bad);
       }

@@ -88,7 +88,7 @@ def compare_tree(r, g_path, g_tau, g_bonus, g_p=None, g_stats=None):
         out["why"].append(f"path gpu {path} (tau {g_tau}) oracle {r['path']} (tau {r['tau']})")
         return out
     if g_stats is not None:
-        got = [int(x) for x in np.asarray(g_stats)]
+        got = [int(x) for x in np.asarray(g_stats)][:4]   # the fifth is path-dependent
         if g_p is not None:
             gp = np.asarray(g_p, dtype=np.float64)
             got[0] -= int(((gp > 0) & (gp < P_EQ0)).sum())
