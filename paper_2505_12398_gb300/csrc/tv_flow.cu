@@ -40,6 +40,7 @@
 #include <stdint.h>
 
 #include <algorithm>
+#include <mutex>
 
 #include "tv_control.cuh"
 #include "tv_device.cuh"
@@ -1288,24 +1289,61 @@ FlowPlan tv_flow_plan(int R, int smem_per_sm, int smem_per_block, int force_ncw,
   return p;
 }
 
+namespace {
+
+// Per device and kernel variant: the dynamic shared memory limit already set
+// and the CTAs per SM for the last size asked (attribute and occupancy
+// queries cost far more host time than the launch itself).
+struct LaunchCache {
+  size_t smem_set = 0;
+  size_t occ_smem = 0;
+  int per_sm = 0;
+};
+constexpr int kCacheDevices = 64;
+std::mutex g_launch_mutex;
+LaunchCache g_launch_cache[kCacheDevices][4];
+
+}  // namespace
+
 int tv_launch_flow(const TravArgs& a, FlowArgs f, int logit_is_bf16, const FlowPlan& plan,
                    int sm_count, cudaStream_t stream, cudaEvent_t* ev) {
   using namespace tvk::flow;
   const size_t smem = plan.smem;
   int stages = plan.stages;
+  int device = 0;
+  if (cudaGetDevice(&device) != cudaSuccess || device < 0 || device >= kCacheDevices) {
+    cudaGetLastError();
+    return -5;
+  }
   if (ev) {
     for (int k = 0; k < 3; ++k)
       if (cudaEventRecord(ev[k], stream) != cudaSuccess) return -5;
   }
-  auto run = [&](auto kernel, int threads) -> int {
-    if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
-        cudaSuccess)
-      return -5;
+  auto run = [&](auto kernel, int threads, int variant) -> int {
     int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, threads, smem) !=
-            cudaSuccess ||
-        per_sm < 1)
-      return -5;
+    {
+      std::lock_guard<std::mutex> lock(g_launch_mutex);
+      LaunchCache& c = g_launch_cache[device][variant];
+      if (smem > c.smem_set) {
+        if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)smem) != cudaSuccess) {
+          cudaGetLastError();
+          return -5;
+        }
+        c.smem_set = smem;
+      }
+      if (c.occ_smem != smem || c.per_sm < 1) {
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&c.per_sm, kernel, threads, smem) !=
+            cudaSuccess) {
+          cudaGetLastError();
+          c.per_sm = 0;
+          return -5;
+        }
+        c.occ_smem = smem;
+      }
+      per_sm = c.per_sm;
+    }
+    if (per_sm < 1) return -5;
     const int grid = per_sm * sm_count;
     if (grid > kMaxGrid) return -5;
     void* params[] = {const_cast<TravArgs*>(&a), &f, &stages};
@@ -1318,11 +1356,13 @@ int tv_launch_flow(const TravArgs& a, FlowArgs f, int logit_is_bf16, const FlowP
   };
   int rc;
   if (plan.ncw == 8)
-    rc = logit_is_bf16 ? run(tv_flow_kernel<tvk::Bf16Logits, 8>, Shape<tvk::Bf16Logits, 8>::kThreads)
-                       : run(tv_flow_kernel<tvk::F32Logits, 8>, Shape<tvk::F32Logits, 8>::kThreads);
+    rc = logit_is_bf16
+             ? run(tv_flow_kernel<tvk::Bf16Logits, 8>, Shape<tvk::Bf16Logits, 8>::kThreads, 0)
+             : run(tv_flow_kernel<tvk::F32Logits, 8>, Shape<tvk::F32Logits, 8>::kThreads, 1);
   else
-    rc = logit_is_bf16 ? run(tv_flow_kernel<tvk::Bf16Logits, 4>, Shape<tvk::Bf16Logits, 4>::kThreads)
-                       : run(tv_flow_kernel<tvk::F32Logits, 4>, Shape<tvk::F32Logits, 4>::kThreads);
+    rc = logit_is_bf16
+             ? run(tv_flow_kernel<tvk::Bf16Logits, 4>, Shape<tvk::Bf16Logits, 4>::kThreads, 2)
+             : run(tv_flow_kernel<tvk::F32Logits, 4>, Shape<tvk::F32Logits, 4>::kThreads, 3);
   if (rc) return rc;
   if (ev && cudaEventRecord(ev[3], stream) != cudaSuccess) return -5;
   return 0;
