@@ -239,6 +239,133 @@ __device__ inline void post_bonus(const TreeSmem& s, Ctl& ctl, int a) {
   ctl.job.nmask = n;
 }
 
+// ---------------------------------------------------- deciding ahead ----
+//
+// While the pass that rejects child c of node i runs, most of the next step is
+// already fixed.  In the common case -- the next remaining child c2 of i is a
+// leaf -- that step is the test of c2, and with
+//   D = S + (1 - p_i),   X = [alpha M_b0(c2) - beta q(c2)]_+ Z' / q(c2),
+//   alpha = p_i a_i,  beta = p_i b_i + 1/Z_i,  Z' = Z_i - q(c),
+// Eqs. (1)-(3) give c2's rate min(X / D, 1), so c2 is accepted iff u D < X, and
+// the pass that rejects c2 uses alpha1 = alpha / (s_i D), beta' = beta / D + 1/Z'.
+// Only D depends on the pass's S, so the next job can be posted right after
+// S arrives and the state update (control_step_ahead) done afterwards.
+// The other common case -- i has no remaining child -- is the test of i
+// itself with its new rate S / D: i is rejected iff u D >= S, and the pass
+// that then rejects i at its parent g depends only on g's state.
+struct Ahead {
+  int ok;          // 1: the next step is decided from D alone (see mode)
+  int mode;        // 1: test of leaf c2 of i; 2: test of i itself (then a pass at g)
+  int i, c, c2, g, nmask;
+  double omp;      // 1 - p_i
+  double X, ainvs, beta, invZn;
+  float alpha1_g, beta_g, rowmax_g;   // mode 2: the pass at g that rejects i
+};
+
+// S-independent part of the next step, after posting the pass for ctl.pending;
+// the next pass's removed tokens (ascending) go to mtok2.
+__device__ inline void prepare_ahead(const TreeSmem& s, const Ctl& ctl, Ahead& ah,
+                                     int* mtok2) {
+  ah.ok = 0;
+  if (ctl.job.kind != kJobPass) return;
+  const int c = ctl.pending, i = s.par[c];
+  const int c2 = first_alive_child(s, i);
+  if (c2 < 0) {
+    if (i == 0) return;   // the root: the bonus draw follows
+    const int g = s.par[i];
+    // the pass post_pass(s, ctl, g, i) would post (g's state does not change)
+    const double pg = s.p[g];
+    ah.alpha1_g = (float)(pg * s.a[g] * s.invs[g]);
+    ah.beta_g = (float)(pg * s.b[g] + s.invZ[g]);
+    ah.rowmax_g = s.rowm[g];
+    int n = 0;
+    for (int j = s.first[g]; j >= 0; j = s.next[j]) {
+      if (j == i || s.state[j] == kAlive) continue;
+      const int t = s.tok[j];
+      int k = n;
+      while (k > 0 && mtok2[k - 1] > t) {
+        mtok2[k] = mtok2[k - 1];
+        --k;
+      }
+      mtok2[k] = t;
+      ++n;
+    }
+    ah.mode = 2;
+    ah.i = i;
+    ah.c = c;
+    ah.c2 = -1;
+    ah.g = g;
+    ah.nmask = n;
+    ah.omp = 1.0 - s.p[i];
+    ah.ok = 1;
+    return;
+  }
+  if (s.first[c2] >= 0 || !(s.rows[i] > 0.f)) return;
+  const double p = s.p[i], a = s.a[i], b = s.b[i];
+  const double Zn = s.Z[i] - (double)s.gq[c];
+  if (!(Zn > 0.0)) return;
+  const double alpha = p * a, beta = p * b + s.invZ[i];
+  const double X = fmax(alpha * s.mb0[c2] - beta * (double)s.gq[c2], 0.0) * Zn * s.invq[c2];
+  if (!(X > 0.0)) return;
+  int n = 0;
+  for (int j = s.first[i]; j >= 0; j = s.next[j]) {
+    if (j == c2 || s.state[j] == kAlive) continue;
+    const int t = s.tok[j];
+    int k = n;
+    while (k > 0 && mtok2[k - 1] > t) {
+      mtok2[k] = mtok2[k - 1];
+      --k;
+    }
+    mtok2[k] = t;
+    ++n;
+  }
+  ah.i = i;
+  ah.c = c;
+  ah.c2 = c2;
+  ah.nmask = n;
+  ah.omp = 1.0 - p;
+  ah.X = X;
+  ah.ainvs = alpha * s.invs[i];
+  ah.beta = beta;
+  ah.invZn = 1.0 / Zn;
+  ah.mode = 1;
+  ah.g = -1;
+  ah.ok = 1;
+}
+
+// control_step for the pass described by `ah`, with the test of ah.c2 going
+// the way `accept` says (the decision taken ahead, so that the state follows
+// the job already posted).
+__device__ inline void control_step_ahead(const TreeSmem& s, Ctl& ctl, const Ahead& ah,
+                                          bool accept) {
+  apply_rejection(s, ctl, ah.i, ah.c);
+  ctl.pending = -1;
+  if (ah.mode == 2) {
+    ctl.node = ah.i;
+    ctl.n_tests++;
+    s.dbgp[ah.i] = (float)s.p[ah.i];
+    if (accept) {
+      post_bonus(s, ctl, ah.i);
+      return;
+    }
+    s.state[ah.i] = kRejected;
+    post_pass(s, ctl, ah.g, ah.i);
+    return;
+  }
+  double pc = 0.0;
+  child_rate(s, ah.i, ah.c2, &pc);
+  s.p[ah.c2] = pc;
+  ctl.node = ah.c2;
+  ctl.n_tests++;
+  s.dbgp[ah.c2] = (float)pc;
+  if (accept) {
+    post_bonus(s, ctl, ah.c2);
+    return;
+  }
+  s.state[ah.c2] = kRejected;
+  post_pass(s, ctl, ah.i, ah.c2);
+}
+
 // Advances the serial traversal until it needs vocabulary work; posts it.
 __device__ inline void control_step(const TreeSmem& s, Ctl& ctl, const float* __restrict__ u) {
   if (ctl.job.kind == kJobPass) {

@@ -85,6 +85,8 @@ struct Shared {
   StageMeta meta[kMaxStages];
   float2 red[kMaxStages][kMaxNCW];   // per-warp partials of the slice ending in a stage
   Ctl ctl;                           // serial control state of the own tree (owner warp)
+  Ahead ahead;                       // the next step, worked out while a pass runs
+  Job fjob;                          // a job posted from `ahead`
   float2 pbuf[kPBuf];                // the own job's partials, as read by the poll
   int jkind, jrows, jK, jslice, outstanding;
 };
@@ -180,6 +182,7 @@ struct Smem {
   int* mtok;     // [kSlots][R] removed tokens of the held slices
   float* mval;   // [kSlots][R] their stored masses
   float* u;      // [R + 1] the own tree's uniforms
+  int* mtok2;    // [R] removed tokens of the pass worked out ahead
   uint64_t* full_bar;
   uint64_t* empty_bar;
   uint64_t* slot_free;
@@ -616,11 +619,22 @@ __device__ void post_nops(const TravArgs& a, const FlowArgs& f, Reserve spec, in
   nop_tags(f, spec.base, spec.n, lane);
 }
 
+// Reserves the queue slots of a rejection pass of the current size (lane 0;
+// not after a bonus draw, which ends the tree).
+__device__ __forceinline__ void reserve_next(const FlowArgs& f, int V, int B, int posted_kind,
+                                             unsigned done, Reserve& spec) {
+  spec.n = 0;
+  if (posted_kind == kJobBonusLeaf || posted_kind == kJobBonusRes) return;
+  spec.slice = adaptive_slice(f, V, B, false, 1, done);
+  spec.n = (V + spec.slice - 1) / spec.slice;
+  spec.base = atomicAdd(&f.ctr[kCtrTail], (unsigned)spec.n);
+}
+
 // Publishes the own tree's current job (ctl.job) as slice items.  A pass may
 // use the slots reserved in `spec`; otherwise those become "no work" items.
 __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const FlowArgs& f,
-                         int b, int V, int lane, unsigned done, Reserve spec) {
-  const Job& j = sh.ctl.job;
+                         int b, int V, int lane, unsigned done, Reserve spec, const Job& j,
+                         const int* mask_tok, const float* mask_val) {
   const bool stats = (j.kind == kJobStats);
   const int n_rows = stats ? j.n_rows : 1;
   const bool use_spec = spec.n > 0 && j.kind == kJobPass;
@@ -630,8 +644,8 @@ __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const
   const int n = n_rows * K;
   const size_t R = (size_t)f.R;
   for (int q = kFlowInlineMask + lane; q < nmask; q += 32) {   // beyond the inline ones
-    f.job_mtok[b * R + q] = s.mask_tok[q];
-    f.job_mval[b * R + q] = s.mask_val[q];
+    f.job_mtok[b * R + q] = mask_tok[q];
+    f.job_mval[b * R + q] = (j.kind == kJobBonusRes) ? mask_val[q] : 0.f;
   }
   // the job's partial slots start as "not yet"
   for (int q = lane; q < n; q += 32) {
@@ -658,8 +672,8 @@ __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const
   float vk[kFlowInlineMask];
 #pragma unroll
   for (int q = 0; q < kFlowInlineMask; ++q) {
-    tk[q] = (q < nmask) ? s.mask_tok[q] : 0x7fffffff;
-    vk[q] = (q < nmask) ? s.mask_val[q] : 0.f;
+    tk[q] = (q < nmask) ? mask_tok[q] : 0x7fffffff;
+    vk[q] = (q < nmask && j.kind == kJobBonusRes) ? mask_val[q] : 0.f;
   }
   const int4 w3 = make_int4(tk[0], tk[1], tk[2], tk[3]);
   const int4 w4 = make_int4(tk[4], tk[5], tk[6], tk[7]);
@@ -703,6 +717,7 @@ __device__ void owner_new_tree(const TravArgs& a, const TreeSmem& s, Shared& sh,
   const typename L::elem* logits = reinterpret_cast<const typename L::elem*>(a.logits);
   if (lane == 0) {
     sh.outstanding = 0;
+    sh.ahead.ok = 0;
     Ctl& c = sh.ctl;
     c.bad = 0u;
     c.accepted = -1;
@@ -1088,15 +1103,83 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
       wait.reset();
       // after a pass the next job is most often a pass of the same row size:
       // reserve its queue slots now, so that the reservation's round trip
-      // overlaps the combine and the control step
-      if (lane == 0 && sh.jkind == kJobPass) {
-        spec.slice = adaptive_slice(f, V, B, false, 1, done_est);
-        spec.n = (V + spec.slice - 1) / spec.slice;
-        spec.base = atomicAdd(&f.ctr[kCtrTail], (unsigned)spec.n);
-      }
+      // overlaps the combine.  (Reserving earlier, while the job runs, holds
+      // fetchers on slots that stay unpublished for microseconds.)
+      if (lane == 0 && sh.jkind == kJobPass) reserve_next(f, V, B, kJobPass, done_est, spec);
       // the bonus draw reads tiles written before its partials
       if (sh.jkind == kJobBonusLeaf || sh.jkind == kJobBonusRes) fence_gpu();
       __syncwarp();
+      if (sh.jkind == kJobPass && sh.ahead.ok && sh.outstanding <= kPBuf) {
+        // ---- the next step was worked out ahead: decide, post, then update ----
+        float S_pass = 0.f;
+        for (int k2 = lane; k2 < sh.jK; k2 += 32) S_pass += sh.pbuf[k2].x;
+        S_pass = warp_sum(S_pass);
+        int fast = 0, post_first = 0, accept = 0;
+        if (lane == 0) {
+          const Ahead& ah = sh.ahead;
+          const double S = (double)S_pass + s.p[ah.i] * sh.ctl.masked_sum;
+          if (S > 1e-300) {
+            fast = 1;
+            const double D = S + ah.omp;
+            Job& jf = sh.fjob;
+            jf.n_rows = 1;
+            if (ah.mode == 1) {
+              accept = ((double)m.u[ah.c2] * D < ah.X) ? 1 : 0;
+              post_first = 1;
+              if (accept) {
+                jf.kind = kJobBonusLeaf;
+                jf.node = ah.c2;
+                jf.nmask = 0;
+              } else {
+                const double invD = 1.0 / D;
+                jf.kind = kJobPass;
+                jf.node = ah.i;
+                jf.nmask = ah.nmask;
+                jf.alpha1 = (float)(ah.ainvs * invD);
+                jf.beta = (float)(ah.beta * invD + ah.invZn);
+                jf.rowmax = s.rowm[ah.i];
+              }
+            } else {
+              accept = ((double)m.u[ah.i] * D < S) ? 1 : 0;
+              if (!accept) {   // the pass at g that rejects i is known already
+                post_first = 1;
+                jf.kind = kJobPass;
+                jf.node = ah.g;
+                jf.nmask = ah.nmask;
+                jf.alpha1 = ah.alpha1_g;
+                jf.beta = ah.beta_g;
+                jf.rowmax = ah.rowmax_g;
+              }
+            }
+            sh.ctl.S = S_pass;
+          }
+        }
+        fast = __shfl_sync(0xffffffffu, fast, 0);
+        if (fast) {
+          post_first = __shfl_sync(0xffffffffu, post_first, 0);
+          accept = __shfl_sync(0xffffffffu, accept, 0);
+          spec.base = __shfl_sync(0xffffffffu, spec.base, 0);
+          spec.n = __shfl_sync(0xffffffffu, spec.n, 0);
+          spec.slice = __shfl_sync(0xffffffffu, spec.slice, 0);
+          __syncwarp();
+          if (post_first) {
+            post_job(s, sh, a, f, my_tree, V, lane, __shfl_sync(0xffffffffu, done_est, 0),
+                     spec, sh.fjob, m.mtok2, s.mask_val);
+            if (lane == 0) control_step_ahead(s, sh.ctl, sh.ahead, accept != 0);
+          } else {
+            if (lane == 0) control_step_ahead(s, sh.ctl, sh.ahead, accept != 0);
+            __syncwarp();
+            post_job(s, sh, a, f, my_tree, V, lane, __shfl_sync(0xffffffffu, done_est, 0),
+                     spec, sh.ctl.job, s.mask_tok, s.mask_val);
+          }
+          spec.n = 0;
+          if (lane == 0) {
+            done_est = ld_relaxed_u32(&f.ctr[kCtrDone]);
+            prepare_ahead(s, sh.ctl, sh.ahead, m.mtok2);   // for the job just posted
+          }
+          continue;
+        }
+      }
       owner_combine<L>(a, f, s, sh, m.u, my_tree, lane);
     }
     spec.base = __shfl_sync(0xffffffffu, spec.base, 0);
@@ -1122,9 +1205,13 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
           st_relaxed_u64(&f.items[q].tag, (f.epoch << 32) | q | kExitTag);
       }
     } else {
-      post_job(s, sh, a, f, my_tree, V, lane, __shfl_sync(0xffffffffu, done_est, 0), spec);
+      post_job(s, sh, a, f, my_tree, V, lane, __shfl_sync(0xffffffffu, done_est, 0), spec,
+               sh.ctl.job, s.mask_tok, s.mask_val);
       spec.n = 0;
-      if (lane == 0) done_est = ld_relaxed_u32(&f.ctr[kCtrDone]);   // used at the next job
+      if (lane == 0) {
+        done_est = ld_relaxed_u32(&f.ctr[kCtrDone]);   // used at the next job
+        prepare_ahead(s, sh.ctl, sh.ahead, m.mtok2);    // while this job runs
+      }
     }
   }
 }
@@ -1152,6 +1239,7 @@ __global__ void __launch_bounds__(Shape<L, kNCW>::kThreads, 16 / kNCW)
   m.mtok = reinterpret_cast<int*>(tree_base + ((tree_smem_bytes_nt(R, 0) + 15) & ~(size_t)15));
   m.mval = reinterpret_cast<float*>(m.mtok + kSlots * R);
   m.u = m.mval + kSlots * R;
+  m.mtok2 = reinterpret_cast<int*>(m.u + R + 1);
   m.full_bar = full_bar;
   m.empty_bar = empty_bar;
   m.slot_free = slot_free;
@@ -1226,7 +1314,7 @@ size_t up256(size_t n) { return (n + 255) & ~static_cast<size_t>(255); }
 size_t flow_smem_bytes(int R, int ncw, int stages) {
   return (size_t)stages * tvk::fused::stage_bytes(ncw) +
          ((tvk::fused::tree_smem_bytes_nt(R, 0) + 15) & ~(size_t)15) +
-         (size_t)tvk::flow::kSlots * R * 8 + (size_t)(R + 1) * 4 + 64;
+         (size_t)tvk::flow::kSlots * R * 8 + (size_t)(R + 1) * 4 + (size_t)R * 4 + 64;
 }
 
 }  // namespace
