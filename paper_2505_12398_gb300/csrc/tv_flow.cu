@@ -382,7 +382,55 @@ __device__ void consumer_role(const TravArgs& a, const FlowArgs& f, const Smem& 
     const char* buf = m.ring + (size_t)stage * S::kStageBytes;
     const E* lb = reinterpret_cast<const E*>(buf);
     const float* qb = reinterpret_cast<const float*>(buf + (size_t)S::kPairElems * S::kLB);
-    for (int t0 = wid * kTileElems; t0 < n; t0 += S::kSweep) {
+    bool done_stage = false;
+    if constexpr (S::kLB == 2) {
+      if (kind == kJobStats) {
+        // Row normaliser, bf16: this warp's maximum over its part of the stage
+        // first (exact on bf16 pairs, after the same clamp as the sums), so
+        // that the running sum is rescaled at most once per stage, then the
+        // sum of e(x) relative to it.  exp2_corrected is used here as in the
+        // passes: its small uniform bias then cancels in alpha1 e(x) = p a e(x)/s.
+        const uint32_t lo_clamp = 0xC61CC61Cu;   // two bf16 -9984
+        __nv_bfloat162 hm = *reinterpret_cast<const __nv_bfloat162*>(&lo_clamp);
+        for (int t0 = wid * kTileElems; t0 < n; t0 += S::kSweep) {
+          const int e0 = t0 + lane * kChunk;
+          if (e0 < n) {
+            const uint4 w = lds128(lb + e0);
+            hm = __hmax2(hm, *reinterpret_cast<const __nv_bfloat162*>(&w.x));
+            hm = __hmax2(hm, *reinterpret_cast<const __nv_bfloat162*>(&w.y));
+            hm = __hmax2(hm, *reinterpret_cast<const __nv_bfloat162*>(&w.z));
+            hm = __hmax2(hm, *reinterpret_cast<const __nv_bfloat162*>(&w.w));
+          }
+        }
+        const uint32_t hb = *reinterpret_cast<uint32_t*>(&hm);
+        const float stage_m =
+            warp_max(fmaxf(__uint_as_float(hb << 16), __uint_as_float(hb & 0xffff0000u)));
+        if (stage_m > m_run) {
+          if (m_run != TV_NEG_INF) {
+            const float sc = L::exp_rel(m_run, stage_m, c_hi, c_lo);
+            acc.s *= sc;
+            acc.c *= sc;
+          }
+          m_run = stage_m;
+        }
+        const float2 mm = make_float2(-m_run, -m_run);
+        for (int t0 = wid * kTileElems; t0 < n; t0 += S::kSweep) {
+          const int e0 = t0 + lane * kChunk;
+          if (e0 < n) {
+            float2 vp[4];
+            bf16x8_pairs(lds128(lb + e0), vp);
+            float2 e[4];
+#pragma unroll
+            for (int k2 = 0; k2 < 4; ++k2)
+              e[k2] = exp2_corrected_x2(__fadd2_rn(vp[k2], mm), ch, cl);
+            const float2 s2 = __fadd2_rn(__fadd2_rn(e[0], e[1]), __fadd2_rn(e[2], e[3]));
+            acc.add(s2.x + s2.y);
+          }
+        }
+        done_stage = true;
+      }
+    }
+    for (int t0 = wid * kTileElems; !done_stage && t0 < n; t0 += S::kSweep) {
       const int e0 = t0 + lane * kChunk;
       const bool valid = e0 < n;
       const int xg = x + e0;
