@@ -382,7 +382,7 @@ def cpu_baseline(inp, args, B):
             # one probe tree per worker to size the sample to the time budget
             t_probe, n_probe = time_oracle(sdir, n_sample, inp.temperature, pool)
             per_round = max(t_probe, 1e-3)
-            reps = max(1, min(50, int(args.cpu_seconds / per_round)))
+            reps = max(1, min(5000, int(args.cpu_seconds / per_round)))
             t, n = time_oracle(sdir, n_sample, inp.temperature, pool, reps=reps)
     return {"value": round(n / t, 4), "unit": "trees/s", "cores": cores, "kind": "oracle",
             "sample": f"{n} oracle tree verifications ({n_sample} distinct trees of the same "
