@@ -49,6 +49,64 @@ def parse_args():
     return ap.parse_args()
 
 
+# ------------------------------------------------------ multi-rank ---------
+#
+# Trees are independent, so N ranks (one GPU each) verify N batches of their
+# own (weak scaling, no collective on the data path).  The only exchanges are
+# the barriers around the timed region and the max-reduction of its length.
+
+def rank_seed(seed, rank):
+    """Input seed of a rank: every rank draws a different batch."""
+    return seed + 7919 * rank
+
+
+def max_over_ranks(value, world, device):
+    """The largest of the ranks' values (the slowest rank sets the job time)."""
+    if world <= 1:
+        return float(value)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank, world, repeats, total_ms):
+    """Units verified by all ranks per second, over `repeats` timed calls."""
+    return units_per_rank * world * repeats / (total_ms / 1e3)
+
+
+# sources of the persistent kernel, in the order its profile's hash covers them
+FLOW_SOURCES = ["tv_control.cuh", "tv_device.cuh", "tv_flow.cu", "tv_launch.h", "tv_ptx.cuh"]
+
+
+def kernel_traffic(workload, batch):
+    """DRAM bytes per launch of the persistent kernel from the committed ncu
+    summary of this workload, or None when there is none or the kernel's
+    sources have changed since it was taken."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", f"launches_{workload}_B{batch}_persistent.md")
+    if not os.path.exists(path):
+        return None
+    fields = {}
+    with open(path) as f:
+        for line in f:
+            key, sep, val = line.strip().partition(":")
+            if sep and key in ("kernel-sources-sha256", "dram-bytes-per-launch"):
+                fields[key] = val.strip()
+    if len(fields) != 2:
+        return None
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2505_12398_gb300", "csrc")
+    for name in FLOW_SOURCES:
+        h.update(name.encode())
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(f.read())
+    if h.hexdigest() != fields["kernel-sources-sha256"]:
+        return None
+    return int(fields["dram-bytes-per-launch"])
+
+
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -205,7 +263,7 @@ def main():
     build()
 
     w = get_workload(args.workload, batch=args.batch, sigma=args.sigma)
-    inp = make_inputs(w, seed=args.seed + 7919 * rank, device=dev)
+    inp = make_inputs(w, seed=rank_seed(args.seed, rank), device=dev)
     B, R = inp.parents.shape
     N, V = R - 1, w.vocab
     lb = 2 if inp.logits.dtype == torch.bfloat16 else 4
@@ -262,10 +320,7 @@ def main():
     clocks = sampler.stop()
     step_ms = [e0[k].elapsed_time(e1[k]) for k in range(args.steps)]
     total_ms = sum(step_ms)
-    t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    total_ms_max = float(t.item())
+    total_ms_max = max_over_ranks(total_ms, world, dev)
     v.set_phase_timing(False)
 
     # end to end through the public API from pinned host buffers
@@ -290,13 +345,11 @@ def main():
         x1.record(stream)
         torch.cuda.synchronize(dev)
         e_ms = x0.elapsed_time(x1)
-        te = torch.tensor([e_ms], dtype=torch.float64, device=dev)
-        if world > 1:
-            dist.all_reduce(te, op=dist.ReduceOp.MAX)
+        e_ms_max = max_over_ranks(e_ms, world, dev)
         h2d = sum(x.numel() * x.element_size() for x in hp)
         d2h = sum(x.numel() * x.element_size() for x in hout)
         assert torch.equal(hout[1], out[1].cpu()), "host entry point disagrees"
-        e2e = {"value": round(B * world * ks / (float(te.item()) / 1e3), 3), "unit": "trees/s",
+        e2e = {"value": round(whole_job_rate(B, world, ks, e_ms_max), 3), "unit": "trees/s",
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": ks}
 
     # CPU baseline: the oracle on host cores, bounded sample of the same batch
@@ -318,8 +371,9 @@ def main():
         kbytes = [0, 0, a_bytes]
         launches_per_step = 1
     dom = max(range(3), key=lambda i: ph[i])
+    traffic = kernel_traffic(w.name, B) if path_code == 2 else None
     ms_step = total_ms_max / args.steps
-    trees_s = B * world * args.steps / (total_ms_max / 1e3)
+    trees_s = whole_job_rate(B, world, args.steps, total_ms_max)
     step_gbs = a_bytes / (ms_step / 1e3) / 1e9
     dom_gbs = kbytes[dom] / (ph[dom] / 1e3) / 1e9 if ph[dom] > 0 else 0.0
     line = {
@@ -355,7 +409,7 @@ def main():
         "roofline": {"bound": "hbm", "kernel": names[dom], "achieved": round(dom_gbs, 2),
                      "peak": peak, "unit": "GB/s", "frac": round(dom_gbs / peak, 4),
                      "peak_kind": peak_kind, "bytes_per_launch": kbytes[dom],
-                     "traffic": None},
+                     "traffic": traffic},
         "roofline_step": {"bound": "hbm", "achieved": round(step_gbs, 2), "peak": peak,
                           "unit": "GB/s", "frac": round(step_gbs / peak, 4)},
         "e2e": e2e,
@@ -379,7 +433,9 @@ def cpu_baseline(inp, args, B):
         sdir = dump_sample(inp, range(n_sample), td)
         ctx = mp.get_context("spawn")
         with ctx.Pool(cores) as pool:
-            # one probe tree per worker to size the sample to the time budget
+            # one probe tree per worker to size the sample to the time budget,
+            # after an untimed round that starts the workers and loads the arrays
+            time_oracle(sdir, n_sample, inp.temperature, pool)
             t_probe, n_probe = time_oracle(sdir, n_sample, inp.temperature, pool)
             per_round = max(t_probe, 1e-3)
             reps = max(1, min(5000, int(args.cpu_seconds / per_round)))
