@@ -55,11 +55,15 @@ def outcome_law(parents, tokens, target_row, draft_row, vocab, root_rate=None,
 
 
 def z_law(parents, mb_table, ms_table, vocab, root_rate=None,
-          with_replacement=False):
+          with_replacement=False, outcome=None):
     """Law of Z^{gamma_max} (Lemma 1) averaged over the draft trees of the
     shape ``parents``: Z = X^tau if tau = gamma_max, else (X^tau, Y, Z_{>tau+1})
     with the tail drawn from the target model.  Keys are token tuples (root
-    excluded); the key None collects the mass where the root was rejected."""
+    excluded); the key None collects the mass where the root was rejected.
+    ``outcome`` is the verifier's exact outcome law on one tree (default:
+    Traversal Verification's ``outcome_law``; the token-level verifier's has
+    the same signature)."""
+    outcome = outcome_law if outcome is None else outcome
     n = len(parents)
     depth = [0] * n
     for i in range(1, n):
@@ -81,7 +85,7 @@ def z_law(parents, mb_table, ms_table, vocab, root_rate=None,
                                               with_replacement=with_replacement):
         total += prob
         pre = node_prefixes(parents, tokens)
-        out = outcome_law(parents, tokens,
+        out = outcome(parents, tokens,
                           target_row=lambda i: mb_table[pre[i]].copy(),
                           draft_row=lambda i: ms_table[pre[i]].copy(),
                           vocab=vocab, root_rate=root_rate,

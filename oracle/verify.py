@@ -126,11 +126,13 @@ def algorithmic_bytes(result, vocab, logit_bytes):
 
 
 def verify_batch(parents, tokens, logits, draft_probs, temperature, uniforms,
-                 trees=None, keep_cdf=False):
+                 trees=None, keep_cdf=False, tree_fn=None):
     """Batch driver: arrays [B, N+1], [B, N+1], [B, N+1, V], [B, N+1, V],
     scalar, [B, N+2].  Invalid trees get tau = -1, bonus = -1 and an all -1
     path, the same marking the library uses.  ``trees`` restricts the work to a
-    subset of tree indices (others are left marked -2)."""
+    subset of tree indices (others are left marked -2).  ``tree_fn`` is the
+    per-tree verifier (default: Traversal Verification, ``verify_tree``)."""
+    tree_fn = verify_tree if tree_fn is None else tree_fn
     parents = np.asarray(parents)
     B, n = parents.shape
     out_path = np.full((B, max(n - 1, 0)), -1, dtype=np.int32)
@@ -140,8 +142,8 @@ def verify_batch(parents, tokens, logits, draft_probs, temperature, uniforms,
     idx = range(B) if trees is None else trees
     for b in idx:
         try:
-            r = verify_tree(parents[b], tokens[b], logits[b], draft_probs[b],
-                            temperature, uniforms[b], keep_cdf=keep_cdf)
+            r = tree_fn(parents[b], tokens[b], logits[b], draft_probs[b],
+                        temperature, uniforms[b], keep_cdf=keep_cdf)
         except InvalidTree as e:
             out_tau[b] = -1
             out_bonus[b] = -1
