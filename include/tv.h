@@ -69,8 +69,8 @@ enum {
   TV_STATUS_BAD_ROW = 64u      /* a target row the traversal needed has no finite logit */
 };
 
-/* Flags for tv_create.  At most one may be given; with none the library picks
-   the path (the persistent kernel when V % 8 == 0, else the three-kernel
+/* Flags for tv_create.  At most one path flag may be given; with none the
+   library picks the path (the persistent kernel when V % 8 == 0, else the three-kernel
    path).  All paths compute the same results; the two single-kernel paths read
    rows with bulk copies and need V % 8 == 0, other vocabularies always take
    the three-kernel path. */
@@ -85,7 +85,19 @@ enum {
   /* One persistent cooperative kernel: each tree's serial control runs in an
      owner CTA, and the vocabulary work of every step is cut into slices that
      any CTA of the grid may process (load balancing across trees). */
-  TV_FLAG_PERSISTENT = 4u
+  TV_FLAG_PERSISTENT = 4u,
+  /* Method, combinable with TV_FLAG_CLUSTER or TV_FLAG_PERSISTENT (or none):
+     token-level tree verification instead of Traversal Verification -- the
+     top-down verifier the paper compares with (§2.2; "Tok.V" in §4).  At the
+     current node (the root first) the children are tried in order by
+     Recursive Rejection Sampling without replacement (Algorithm 2); an
+     accepted child becomes the current node; the bonus token comes from an
+     accepted leaf's row or from the residual once every child of the current
+     node is rejected.  Same arguments, outputs and uniforms convention.
+     Needs a single-kernel path: tv_create returns TV_ERR_INVALID_ARG with
+     TV_FLAG_UNFUSED or when V % 8 != 0, and a call that could only run the
+     three-kernel path returns TV_ERR_INVALID_ARG. */
+  TV_FLAG_TOKEN_LEVEL = 8u
 };
 
 /*
@@ -98,7 +110,7 @@ enum {
  *   max_batch  : largest B later calls may pass; >= 1.
  *   logit_dtype: element type of target_logits in later calls.
  *   flags      : TV_FLAG_NONE or one of TV_FLAG_UNFUSED, TV_FLAG_CLUSTER,
- *                TV_FLAG_PERSISTENT.
+ *                TV_FLAG_PERSISTENT, optionally ORed with TV_FLAG_TOKEN_LEVEL.
  * Errors: TV_ERR_INVALID_ARG, TV_ERR_VOCAB, TV_ERR_CUDA, TV_ERR_DEVICE.
  */
 int tv_create(tv_handle** out, int device, int vocab, int max_nodes, int max_batch,

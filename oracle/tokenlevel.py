@@ -37,8 +37,8 @@ from collections import defaultdict
 
 import numpy as np
 
-from .traversal import (InvalidTree, _condition, _one_like, acceptance_rate, draft_without,
-                        residual_mass, residual_target, validate_tree)
+from .traversal import (InvalidTree, _cancellation, _condition, _one_like, acceptance_rate,
+                        draft_without, residual_mass, residual_target, validate_tree)
 from .verify import inverse_cdf, softmax_f64, verify_batch
 
 
@@ -103,6 +103,11 @@ class TokenLevelState:
         self.passes[self.node] += 1
         self.kappa.append(_condition(self.one, self.mb, self.ms, S))
         if S > 0:
+            # instrumentation: cancellation in the residual of every sibling
+            # still to be tested, on top of that of S
+            for d in self.children[self.node][self.next + 1:]:
+                x = self.tokens[d]
+                self.kappa.append(self.kappa[-1] + _cancellation(self.mb[x], self.ms[x]))
             self.mb = residual_target(self.one, self.mb, self.ms, S)
         else:
             self.degenerate += 1

@@ -9,6 +9,9 @@ TV_BF16 = 0
 TV_FP32 = 1
 # tv_create flags: which kernel path a handle uses ("auto" lets the library pick)
 PATH_FLAGS = {"auto": 0, "three": 1, "cluster": 2, "persistent": 4}
+# tv_create flags: the verification method ("token": the top-down token-level
+# verifier the paper compares with; single-kernel paths only)
+METHOD_FLAGS = {"traversal": 0, "token": 8}
 TV_STATUS = {
     "BAD_TREE": 1,
     "BAD_TOKEN": 2,
@@ -97,7 +100,8 @@ class Verifier:
     the handle's device with the dtypes and layouts of include/tv.h.
     """
 
-    def __init__(self, vocab, max_nodes, max_batch, logit_dtype="bf16", device=0, path="auto"):
+    def __init__(self, vocab, max_nodes, max_batch, logit_dtype="bf16", device=0, path="auto",
+                 method="traversal"):
         import torch
         self.lib = library()
         if logit_dtype in ("bf16", torch.bfloat16, TV_BF16):
@@ -111,8 +115,12 @@ class Verifier:
         h = ctypes.c_void_p()
         if path not in PATH_FLAGS:
             raise ValueError(f"unknown path {path!r}; one of {sorted(PATH_FLAGS)}")
+        if method not in METHOD_FLAGS:
+            raise ValueError(f"unknown method {method!r}; one of {sorted(METHOD_FLAGS)}")
+        self.method = method
         rc = self.lib.tv_create(ctypes.byref(h), self.device.index or 0, vocab, max_nodes,
-                                max_batch, self.dtype_code, PATH_FLAGS[path])
+                                max_batch, self.dtype_code,
+                                PATH_FLAGS[path] | METHOD_FLAGS[method])
         if rc != 0:
             raise LibraryError("tv_create", rc, self.lib)
         self.handle = h

@@ -139,12 +139,15 @@ int verify_impl(tv_handle* h, int B, int N, const int32_t* parents, const int32_
   a.out_node_p = out_node_p;
   a.out_stats = out_stats;
   a.status = h->status;
+  a.token_level = (h->flags & TV_FLAG_TOKEN_LEVEL) ? 1 : 0;
   const int rows = B * (N + 1);
   int grid = h->sm_count * 4;
   if (grid > rows) grid = rows;
   if (grid < 1) grid = 1;
   FusedPlan plan;
   const Path path = choose_path(h, B, N + 1, &plan);
+  // the three-kernel path implements Traversal Verification only
+  if (path == kPathThree && a.token_level) return TV_ERR_INVALID_ARG;
   const int bf16 = h->dtype == TV_BF16 ? 1 : 0;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   cudaEvent_t* ev = h->timing ? h->ev : nullptr;
@@ -175,7 +178,12 @@ int tv_create(tv_handle** out, int device, int vocab, int max_nodes, int max_bat
   if (vocab < 1 || vocab > kMaxVocab) return TV_ERR_VOCAB;
   if (max_nodes < 0 || max_nodes + 1 > kMaxRows || max_batch < 1) return TV_ERR_INVALID_ARG;
   if (logit_dtype != TV_BF16 && logit_dtype != TV_FP32) return TV_ERR_INVALID_ARG;
-  if ((flags & ~kPathFlags) || __builtin_popcount(flags) > 1) return TV_ERR_INVALID_ARG;
+  if ((flags & ~(kPathFlags | TV_FLAG_TOKEN_LEVEL)) ||
+      __builtin_popcount(flags & kPathFlags) > 1)
+    return TV_ERR_INVALID_ARG;
+  // the token-level method runs on the single-kernel paths only
+  if ((flags & TV_FLAG_TOKEN_LEVEL) && ((flags & TV_FLAG_UNFUSED) || (vocab % 8) != 0))
+    return TV_ERR_INVALID_ARG;
   int ndev = 0;
   if (cudaGetDeviceCount(&ndev) != cudaSuccess || device < 0 || device >= ndev) {
     cudaGetLastError();

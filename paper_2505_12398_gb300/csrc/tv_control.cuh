@@ -415,5 +415,72 @@ __device__ inline void control_step(const TreeSmem& s, Ctl& ctl, const float* __
   }
 }
 
+// ------------------------------------------- token-level verification ----
+//
+// The top-down verifier Traversal Verification is compared with (§2.2, "Tok.V"
+// of §4): at the current node ctl.node its children are tried in order by
+// Recursive Rejection Sampling without replacement (Algorithm 2).  That is
+// Eqs. (1)-(3) with the node's rate held at 1: min(M_b'(x_c) / M_s'(x_c), 1) is
+// child_rate at p = 1, and the residual update [M_b' - M_s']_+ / S with x_c
+// removed from M_s' is apply_rejection at p = 1, which leaves p = 1.  An
+// accepted child becomes the current node with its own rows (a = 1, b = 0,
+// Z = 1 from the tree set-up); the bonus token comes from an accepted leaf's
+// own row, or from the current node's residual once all its children are
+// rejected.  Only the current node's row is normalised.  A child of rate 0
+// is rejected without counting as a test (its uniform cannot accept it).
+__device__ inline void control_step_token(const TreeSmem& s, Ctl& ctl,
+                                          const float* __restrict__ u) {
+  if (ctl.job.kind == kJobPass) {
+    const int c = ctl.pending, i = s.par[c];
+    apply_rejection(s, ctl, i, c);
+    ctl.pending = -1;
+    ctl.node = i;
+  }
+  for (;;) {
+    const int node = ctl.node;
+    if (s.first[node] < 0) {   // an accepted leaf (or a root without children)
+      post_bonus(s, ctl, node);
+      return;
+    }
+    if (!(s.rows[node] > 0.f)) {
+      ctl.job.kind = kJobStats;
+      ctl.job.n_rows = 1;
+      s.job_rows[0] = node;
+      return;
+    }
+    const int c = first_alive_child(s, node);
+    if (c < 0) {               // every child rejected: the residual at node
+      post_bonus(s, ctl, node);
+      return;
+    }
+    double pc;
+    if (!child_rate(s, node, c, &pc)) {
+      ctl.bad |= 8u;
+      ctl.accepted = -1;
+      ctl.job.kind = kJobDone;
+      return;
+    }
+    s.dbgp[c] = (float)pc;
+    if (pc > 0.0) {
+      ctl.n_tests++;
+      if ((double)u[c] < pc) {   // accepted: c becomes the current node
+        s.p[c] = 1.0;
+        ctl.node = c;
+        continue;
+      }
+    }
+    s.state[c] = kRejected;
+    post_pass(s, ctl, node, c);
+    return;
+  }
+}
+
+// One step of the tree's verification method until it needs vocabulary work.
+__device__ inline void advance(const TreeSmem& s, Ctl& ctl, const float* __restrict__ u,
+                               bool token_level) {
+  if (token_level) control_step_token(s, ctl, u);
+  else control_step(s, ctl, u);
+}
+
 }  // namespace fused
 }  // namespace tvk

@@ -833,7 +833,7 @@ __device__ void owner_new_tree(const TravArgs& a, const TreeSmem& s, Shared& sh,
     sh.ctl.bad = bad;
     if (bad == 0u) {
       s.p[0] = 1.0;
-      control_step(s, sh.ctl, u);
+      advance(s, sh.ctl, u, a.token_level != 0);
     } else {
       sh.ctl.job.kind = kJobDone;
     }
@@ -1052,7 +1052,7 @@ __device__ void owner_combine(const TravArgs& a, const FlowArgs& f, const TreeSm
   __syncwarp();
   if (lane == 0 && sh.ctl.job.kind != kJobDone) {
     if (sh.ctl.bad & 64u) sh.ctl.job.kind = kJobDone;
-    else control_step(s, sh.ctl, u);
+    else advance(s, sh.ctl, u, a.token_level != 0);
   }
   __syncwarp();
 }
@@ -1223,7 +1223,8 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
           spec.n = 0;
           if (lane == 0) {
             done_est = ld_relaxed_u32(&f.ctr[kCtrDone]);
-            prepare_ahead(s, sh.ctl, sh.ahead, m.mtok2);   // for the job just posted
+            if (a.token_level) sh.ahead.ok = 0;            // (Traversal Verification only)
+            else prepare_ahead(s, sh.ctl, sh.ahead, m.mtok2);   // for the job just posted
           }
           continue;
         }
@@ -1258,7 +1259,8 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
       spec.n = 0;
       if (lane == 0) {
         done_est = ld_relaxed_u32(&f.ctr[kCtrDone]);   // used at the next job
-        prepare_ahead(s, sh.ctl, sh.ahead, m.mtok2);    // while this job runs
+        if (a.token_level) sh.ahead.ok = 0;             // (Traversal Verification only)
+        else prepare_ahead(s, sh.ctl, sh.ahead, m.mtok2);    // while this job runs
       }
     }
   }

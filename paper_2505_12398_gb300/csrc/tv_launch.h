@@ -21,6 +21,7 @@ struct TravArgs {
   float* out_node_p;           // [B][N+1] or nullptr
   int32_t* out_stats;          // [B][4] or nullptr
   uint32_t* status;            // status word (OR of TV_STATUS_* bits)
+  int token_level;             // 1: token-level (top-down) verification instead (fused paths)
 };
 
 // Launch plan of the fused kernel: cluster size, ring stages, shared memory.

@@ -138,6 +138,7 @@ extern "C" int tv_verify_batch_noalloc(int device, int B, int N, int vocab, tv_d
       a.out_node_p = nullptr;
       a.out_stats = nullptr;
       a.status = status;
+      a.token_level = 0;
       const int rows = B * (N + 1);
       int grid = g_sm_count[device] * 4;
       if (grid > rows) grid = rows;

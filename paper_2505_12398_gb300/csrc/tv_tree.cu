@@ -219,7 +219,7 @@ __global__ void __launch_bounds__(NCW * 32 + 32, 16 / NCW) tv_tree_kernel(TravAr
     for (;;) {
       if (tid == 0) {
         if (*vbad & (32u | 64u)) ctl.job.kind = kJobDone;         // timeout / unusable row
-        else if (ctl.job.kind != kJobDone) control_step(s, ctl, u);
+        else if (ctl.job.kind != kJobDone) advance(s, ctl, u, args.token_level != 0);
       }
       named_sync(1, kThreads);
       const Job job = ctl.job;

@@ -28,7 +28,7 @@ def tv():
     return tv
 
 
-def z_counts(tv, shape, V, count, seed, wrong_target=False):
+def z_counts(tv, shape, V, count, seed, wrong_target=False, method="traversal"):
     rng = np.random.default_rng(seed)
     L = 4
     tb = float_table(V, L, seed, concentration=0.8)
@@ -55,7 +55,7 @@ def z_counts(tv, shape, V, count, seed, wrong_target=False):
     dp = torch.from_numpy(drafts).to(dev)
     un = torch.rand(count, n + 1, generator=torch.Generator(device=dev).manual_seed(seed),
                     device=dev)
-    v = tv.Verifier(V, n - 1, count, "fp32")
+    v = tv.Verifier(V, n - 1, count, "fp32", method=method)
     path, tau, bonus = v.verify(par, tok, lg, dp, 1.0, un)
     torch.cuda.synchronize()
     status = v.status()
@@ -102,3 +102,10 @@ def test_kernel_output_law_is_target(tv, shape, V):
 def test_negative_control_detects_wrong_law(tv):
     obs, exp = z_counts(tv, [-1, 0, 0, 1, 1, 2, 2], 4, 1_000_000, seed=5, wrong_target=True)
     assert chi2_p(obs, exp) < 1e-6
+
+
+@pytest.mark.parametrize("shape", [[-1, 0, 0, 1, 1, 2, 2], [-1, 0, 1, 2]])
+def test_token_level_output_law_is_target(tv, shape):
+    """The token-level verifier (TV_FLAG_TOKEN_LEVEL) is lossless too."""
+    obs, exp = z_counts(tv, shape, 8, 1_000_000, seed=101 + len(shape), method="token")
+    assert chi2_p(obs, exp) > 1e-3
