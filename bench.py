@@ -39,6 +39,9 @@ def parse_args():
     ap.add_argument("--batch", type=int, default=None)
     ap.add_argument("--sigma", type=float, default=None)
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--method", choices=["traversal", "token"], default="traversal",
+                    help="verification method: Traversal Verification, or the token-level "
+                         "(top-down RRS without replacement) verifier it is compared with")
     ap.add_argument("--path", choices=["auto", "persistent", "cluster", "three"], default="auto",
                     help="kernel path of the handle (auto: the library's choice)")
     ap.add_argument("--e2e-steps", type=int, default=10)
@@ -204,16 +207,19 @@ class _DirArrays:
 
 
 def _oracle_dir_worker(args):
-    path, b, temperature = args
-    from oracle.verify import verify_tree
+    path, b, temperature, method = args
+    if method == "token":
+        from oracle.tokenlevel import verify_tree
+    else:
+        from oracle.verify import verify_tree
     d = _DirArrays(path)
     r = verify_tree(d["parents"][b], d["tokens"][b], d["logits"][b], d["drafts"][b],
                     temperature, d["uniforms"][b])
     return r["tau"]
 
 
-def time_oracle(sample_dir, n_trees, temperature, pool, reps=1):
-    jobs = [(sample_dir, b % n_trees, temperature) for b in range(n_trees * reps)]
+def time_oracle(sample_dir, n_trees, temperature, pool, reps=1, method="traversal"):
+    jobs = [(sample_dir, b % n_trees, temperature, method) for b in range(n_trees * reps)]
     t0 = time.perf_counter()
     pool.map(_oracle_dir_worker, jobs, chunksize=1)
     return time.perf_counter() - t0, len(jobs)
@@ -267,7 +273,8 @@ def main():
     B, R = inp.parents.shape
     N, V = R - 1, w.vocab
     lb = 2 if inp.logits.dtype == torch.bfloat16 else 4
-    v = tv.Verifier(V, N, B, "bf16" if lb == 2 else "fp32", device=dev.index, path=args.path)
+    v = tv.Verifier(V, N, B, "bf16" if lb == 2 else "fp32", device=dev.index, path=args.path,
+                    method=args.method)
     stream = torch.cuda.current_stream(dev)
 
     # decisions are a deterministic function of the inputs: one instrumented
@@ -371,7 +378,8 @@ def main():
         kbytes = [0, 0, a_bytes]
         launches_per_step = 1
     dom = max(range(3), key=lambda i: ph[i])
-    traffic = kernel_traffic(w.name, B) if path_code == 2 else None
+    traffic = (kernel_traffic(w.name, B)
+               if path_code == 2 and args.method == "traversal" else None)
     ms_step = total_ms_max / args.steps
     trees_s = whole_job_rate(B, world, args.steps, total_ms_max)
     step_gbs = a_bytes / (ms_step / 1e3) / 1e9
@@ -391,7 +399,7 @@ def main():
         "dtype": "f32",
         "data": "synthetic (seeded logits with Zipf rank prior, noisy-drafter probabilities, "
                 "EAGLE-shaped draft trees sampled without replacement)",
-        "config": {"workload": w.name, "batch": B, "vocab": V, "nodes": N,
+        "config": {"workload": w.name, "batch": B, "vocab": V, "nodes": N, "method": args.method,
                    "normalised_rows_per_tree": round(row_bytes / (V * lb) / B, 3) if B else 0,
                    "logit_dtype": "bf16" if lb == 2 else "fp32",
                    "temperature": w.temperature, "sigma": w.sigma, "seed": args.seed,
@@ -435,11 +443,13 @@ def cpu_baseline(inp, args, B):
         with ctx.Pool(cores) as pool:
             # one probe tree per worker to size the sample to the time budget,
             # after an untimed round that starts the workers and loads the arrays
-            time_oracle(sdir, n_sample, inp.temperature, pool)
-            t_probe, n_probe = time_oracle(sdir, n_sample, inp.temperature, pool)
+            time_oracle(sdir, n_sample, inp.temperature, pool, method=args.method)
+            t_probe, n_probe = time_oracle(sdir, n_sample, inp.temperature, pool,
+                                           method=args.method)
             per_round = max(t_probe, 1e-3)
             reps = max(1, min(5000, int(args.cpu_seconds / per_round)))
-            t, n = time_oracle(sdir, n_sample, inp.temperature, pool, reps=reps)
+            t, n = time_oracle(sdir, n_sample, inp.temperature, pool, reps=reps,
+                               method=args.method)
     return {"value": round(n / t, 4), "unit": "trees/s", "cores": cores, "kind": "oracle",
             "sample": f"{n} oracle tree verifications ({n_sample} distinct trees of the same "
                       f"batch, repeated {reps}x) across {cores} spawn workers, {t:.1f} s"}
@@ -462,10 +472,10 @@ def run_reference(args, world, rank):
         ctx = mp.get_context("spawn")
         with ctx.Pool(cores) as pool:
             for _ in range(args.warmup):
-                time_oracle(sdir, per_step, inp.temperature, pool)
+                time_oracle(sdir, per_step, inp.temperature, pool, method=args.method)
             times = []
             for _ in range(args.steps):
-                t, _ = time_oracle(sdir, per_step, inp.temperature, pool)
+                t, _ = time_oracle(sdir, per_step, inp.temperature, pool, method=args.method)
                 times.append(t)
     total = sum(times)
     value = per_step * args.steps / total
@@ -477,6 +487,7 @@ def run_reference(args, world, rank):
         "warmup": args.warmup, "ms_per_step": round(total / args.steps * 1e3, 3),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": {"workload": w.name, "batch": w.batch, "vocab": w.vocab,
+                                         "method": args.method,
                                          "nodes": w.nodes},
         "cpu_baseline": {"value": round(value, 4), "unit": "trees/s", "cores": cores,
                          "kind": "oracle",
