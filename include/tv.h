@@ -198,6 +198,21 @@ int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
                          void* cuda_stream);
 
 /*
+ * tv_debug_withhold_job -- test hook for the failure path; no counterpart in
+ * the paper.  The next call on this handle that runs the persistent kernel
+ * writes tree `tree`'s first job into the work queue but never publishes it.
+ * The CTAs holding its queue slots and the tree's owner wait on it until the
+ * kernel's idle limit (2 s without progress).  The kernel then raises its abort
+ * flag and every role exits.  That call returns normally, the status word gets
+ * TV_STATUS_TIMEOUT, and every tree not finished by then reports -1
+ * (accept_len, bonus, path).  Later calls on the handle are unaffected.  Calls
+ * on the other paths ignore the request and leave it pending.
+ *   tree : 0 <= tree < the handle's max_batch.
+ * Errors: TV_ERR_INVALID_ARG.
+ */
+int tv_debug_withhold_job(tv_handle* h, int tree);
+
+/*
  * tv_get_status -- synchronise the handle's device and return, in *status, the
  * OR of the TV_STATUS_* bits raised since the previous tv_get_status call
  * (then clear them).  Errors: TV_ERR_INVALID_ARG, TV_ERR_CUDA.

@@ -48,6 +48,7 @@ _SIGS = {
     "tv_verify_batch_debug": (_I, [_P, _I, _I, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P, _P, _P]),
     "tv_verify_batch_host": (_I, [_P, _I, _I, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P]),
     "tv_get_status": (_I, [_P, ctypes.POINTER(ctypes.c_uint32)]),
+    "tv_debug_withhold_job": (_I, [_P, _I]),
     "tv_destroy": (_I, [_P]),
     "tv_set_phase_timing": (_I, [_P, _I]),
     "tv_last_phase_ms": (_I, [_P, ctypes.POINTER(ctypes.c_float)]),
@@ -222,6 +223,13 @@ class Verifier:
         if rc != 0:
             raise LibraryError("tv_launch_shape", rc, self.lib)
         return tuple(o.value for o in out)
+
+    def withhold_job(self, tree):
+        """Test hook (tv_debug_withhold_job): the next persistent-kernel call
+        never publishes tree ``tree``'s first job, so its waits run out."""
+        rc = self.lib.tv_debug_withhold_job(self.handle, int(tree))
+        if rc != 0:
+            raise LibraryError("tv_debug_withhold_job", rc, self.lib)
 
     def status(self):
         """Synchronise and return (and clear) the TV_STATUS_* bits raised."""

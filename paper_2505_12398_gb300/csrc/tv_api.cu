@@ -33,6 +33,7 @@ struct tv_handle {
   void* flow_ws = nullptr;       // persistent kernel's queue and partials
   size_t flow_ws_bytes = 0;
   unsigned long long epoch = 0;  // per-call tag of the persistent kernel's queue
+  int withhold_tree = -1;        // test hook for the next persistent call (-1: none)
   // staging for tv_verify_batch_host (allocated on first use)
   char* stage = nullptr;
   size_t stage_bytes = 0;
@@ -159,6 +160,8 @@ int verify_impl(tv_handle* h, int B, int N, const int32_t* parents, const int32_
     if (tv_flow_bind(h->flow_ws, h->flow_ws_bytes, B, N + 1, h->vocab, fp, &f) != 0)
       return TV_ERR_CAPACITY;
     f.epoch = ++h->epoch;
+    f.withhold_tree = h->withhold_tree;
+    h->withhold_tree = -1;
     rc = tv_launch_flow(a, f, bf16, fp, h->sm_count, st, ev);
   } else {
     rc = tv_launch_all(a, bf16, h->row_list, h->n_rows, grid, st, ev);
@@ -340,6 +343,12 @@ int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
     cudaGetLastError();
     return TV_ERR_CUDA;
   }
+  return TV_OK;
+}
+
+int tv_debug_withhold_job(tv_handle* h, int tree) {
+  if (!h || tree < 0 || tree >= h->max_batch) return TV_ERR_INVALID_ARG;
+  h->withhold_tree = tree;
   return TV_OK;
 }
 

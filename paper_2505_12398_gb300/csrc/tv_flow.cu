@@ -744,8 +744,11 @@ __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const
   }
   fence_gpu();   // bodies, masks and partial resets before tags
   __syncwarp();
-  for (int q = lane; q < n; q += 32)
-    st_relaxed_u64(&f.items[base + q].tag, (f.epoch << 32) | (unsigned long long)(base + q));
+  // (test hook: a withheld tree's job is never published, so the waits on it
+  // run out and the kernel ends through its abort path)
+  if (b != f.withhold_tree)
+    for (int q = lane; q < n; q += 32)
+      st_relaxed_u64(&f.items[base + q].tag, (f.epoch << 32) | (unsigned long long)(base + q));
   if (spec.n > 0 && !use_spec) nop_tags(f, spec.base, spec.n, lane);
   if (lane == 0) {
     sh.outstanding = n;
@@ -1399,6 +1402,7 @@ int tv_flow_bind(void* base, size_t bytes, int B, int R, int V, const FlowPlan& 
   f->slice_pass = plan.slice_pass;
   f->slice_stats = plan.slice_stats;
   f->slice_min = plan.slice_min;
+  f->withhold_tree = -1;
   return (size_t)(p - static_cast<char*>(base)) <= bytes ? 0 : -4;
 }
 

@@ -82,6 +82,7 @@ struct FlowArgs {
   int cap, R, Kmax, ntiles;
   int slice_pass, slice_stats;   // largest tokens per slice (multiples of 256)
   int slice_min;                 // smallest tokens per slice (multiple of 256)
+  int withhold_tree;             // test hook: this tree's jobs are never published (-1: none)
 };
 
 // Launch shape of the persistent kernel.
