@@ -17,6 +17,9 @@ Recipe (all draws seeded, on any torch device):
 * draft probabilities  q[b, i] = softmax((float(l[b, i]) + sigma n) / T),
   n ~ N(0, 1) i.i.d., float32 -- so sigma sets how far the drafter is from
   the target and hence the acceptance rate;
+* workloads: EAGLE-shaped and sweep trees of depth 5-8, and deep768, a
+  Sequoia-scale tree of 768 nodes and depth 24; make_inputs_random_shapes
+  gives a batch of trees that all differ in shape;
 * tree shape from per-level sizes and maximum branching, parents allotted
   greedily to the earliest nodes of the previous level (nodes numbered level
   by level, so parents precede children and the first chain is the deepest);
@@ -74,6 +77,11 @@ def tree_from_levels(levels, branching):
 
 EAGLE_LEVELS = (4, 10, 16, 16, 8, 6)
 EAGLE_BRANCHING = (4, 3, 2, 2, 1, 1)
+# a Sequoia-scale tree (the large, deep trees §4.2 expects larger gains on):
+# 768 draft nodes, depth 24, wide near the root and a long tail of chains
+DEEP768_LEVELS = (4, 8, 16, 32, 48, 64, 64, 64, 64, 64, 64, 56, 40, 32, 28, 24, 20, 16, 16,
+                  12, 12, 8, 8, 4)
+DEEP768_BRANCHING = (4, 2, 2, 2, 2, 2) + (1,) * 18
 
 WORKLOADS = {
     "tiny": Workload("tiny", 1, 64, parents=(-1, 0, 0, 1, 1, 2, 2, 3),
@@ -95,6 +103,8 @@ WORKLOADS = {
                         description="26-node trees, depth 5, V=151936, bf16"),
     "sweep60": Workload("sweep60", 256, 151936, EAGLE_LEVELS, EAGLE_BRANCHING,
                         description="60-node trees, depth 6, V=151936, bf16"),
+    "deep768": Workload("deep768", 64, 32000, DEEP768_LEVELS, DEEP768_BRANCHING,
+                        description="64 Sequoia-scale trees (768 nodes, depth 24), V=32000, bf16"),
     "sweep120": Workload("sweep120", 256, 151936, (4, 12, 24, 24, 20, 16, 12, 8),
                          (4, 3, 2, 1, 1, 1, 1, 1),
                          description="120-node trees, depth 8, V=151936, bf16"),
@@ -176,3 +186,45 @@ def internal_rows(parents):
     for i in range(1, len(parents)):
         has[parents[i]] = True
     return [i for i, h in enumerate(has) if h]
+
+
+def random_parents(nodes, rng, width):
+    """Parent array (row 0 = root) of a random tree with `nodes` draft nodes:
+    node i's parent is drawn uniformly from the `width` nodes before it, so
+    small widths give deep, chain-like trees and large ones bushy trees."""
+    parents = [-1]
+    for i in range(1, nodes + 1):
+        parents.append(int(rng.integers(max(0, i - width), i)))
+    return parents
+
+
+def make_inputs_random_shapes(batch, nodes, vocab, seed=0, device="cpu",
+                              logit_dtype=torch.bfloat16, temperature=1.0, sigma=1.0,
+                              widths=(2, 4, 8, 32)):
+    """A batch whose trees all have different random shapes with the same
+    node count (tree b uses width widths[b % len(widths)] in random_parents);
+    rows, draft probabilities and uniforms as in make_inputs, children drawn
+    from their parent's draft row without replacement."""
+    import numpy as np
+    w = Workload("random_shapes", batch, vocab, parents=tuple([-1] + list(range(nodes))),
+                 logit_dtype=logit_dtype, temperature=temperature, sigma=sigma)
+    inp = make_inputs(w, seed=seed, device=device)
+    dev = inp.logits.device
+    rng = np.random.default_rng(seed + 3000)
+    shapes = [random_parents(nodes, rng, widths[b % len(widths)]) for b in range(batch)]
+    gk = torch.Generator(device=dev).manual_seed(seed + 4000)
+    tokens = torch.zeros(batch, nodes + 1, dtype=torch.int64, device=dev)
+    for b, parents in enumerate(shapes):
+        kids = [[] for _ in range(nodes + 1)]
+        for i in range(1, nodes + 1):
+            kids[parents[i]].append(i)
+        for i, ks in enumerate(kids):
+            if not ks:
+                continue
+            u = torch.rand(vocab, generator=gk, device=dev).clamp_(min=1e-12)
+            keys = torch.log(inp.draft_probs[b, i].clamp(min=1e-38)) - torch.log(-torch.log(u))
+            tokens[b, ks] = torch.topk(keys, len(ks), sorted=True).indices
+    inp.parents = torch.tensor(shapes, dtype=torch.int32, device=dev)
+    inp.tokens = tokens.to(torch.int32).contiguous()
+    inp.meta = {"workload": f"random_shapes_n{nodes}", "seed": seed}
+    return inp
