@@ -198,6 +198,47 @@ int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
                          void* cuda_stream);
 
 /*
+ * tv_lm_head -- the target model's last layer fused with the row normalisers
+ * (the step before verification; not a step of the paper's method itself).
+ * Computes the logits l = H W^T on the tensor cores and, in the same pass,
+ * each stored row's normaliser (max_v l[v], sum_v 2^((l[v] - max) log2(e) / T)),
+ * evaluated on the bf16 values stored.  Given those normalisers,
+ * tv_verify_batch_stats does not stream any row to normalise it.
+ *   M              rows (e.g. B * (N+1) for a batch of trees, rows in the
+ *                  [B][N+1] order of target_logits); M <= max_batch * (max_nodes + 1).
+ *   K              hidden size; K % 64 == 0.
+ *   hidden         [M][K] bf16, 16-byte aligned.
+ *   weight         [V][K] bf16 (output embedding, V = the handle's vocab), 16-byte aligned.
+ *   temperature    > 0, the temperature the normalisers are for.
+ *   out_logits     [M][V] bf16, 16-byte aligned.
+ *   out_row_stats  [M][2] fp32 (max, sum), 8-byte aligned.
+ * The handle must have been created for bf16 logits with V % 8 == 0.  The
+ * first call allocates the handle's per-(row, 256-column tile) scratch for
+ * max_batch * (max_nodes + 1) rows (a later call with a larger vocabulary
+ * cannot happen: V is the handle's).
+ * Errors: TV_ERR_INVALID_ARG, TV_ERR_CAPACITY, TV_ERR_TEMPERATURE, TV_ERR_CUDA.
+ */
+int tv_lm_head(tv_handle* h, int M, int K, const void* hidden, const void* weight,
+               float temperature, void* out_logits, float* out_row_stats, void* cuda_stream);
+
+/*
+ * tv_verify_batch_stats -- tv_verify_batch with the target rows' normalisers
+ * given (row_stats [B][N+1][2] fp32 (max, sum of 2^((l - max) log2(e) / T)) of
+ * the bf16 or fp32 target_logits, as tv_lm_head writes them for the same
+ * temperature), so no row is streamed to normalise it.  out_node_p and
+ * out_stats are optional (NULL) and have the layouts of tv_verify_batch_debug
+ * (out_stats[b][4], rows normalised by this call, is then 0).  Runs on the
+ * persistent kernel only: other paths return TV_ERR_INVALID_ARG.
+ * Errors: those of tv_verify_batch.
+ */
+int tv_verify_batch_stats(tv_handle* h, int B, int N, const int32_t* parents,
+                          const int32_t* draft_tokens, const void* target_logits,
+                          const float* draft_probs, float temperature, const float* uniforms,
+                          const float* row_stats, int32_t* out_accepted_path,
+                          int32_t* out_accept_len, int32_t* out_bonus_token, float* out_node_p,
+                          int32_t* out_stats, void* cuda_stream);
+
+/*
  * tv_debug_withhold_job -- test hook for the failure path; no counterpart in
  * the paper.  The next call on this handle that runs the persistent kernel
  * writes tree `tree`'s first job into the work queue but never publishes it.

@@ -47,6 +47,9 @@ _SIGS = {
     "tv_verify_batch": (_I, [_P, _I, _I, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P]),
     "tv_verify_batch_debug": (_I, [_P, _I, _I, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P, _P, _P]),
     "tv_verify_batch_host": (_I, [_P, _I, _I, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P]),
+    "tv_verify_batch_stats": (_I, [_P, _I, _I, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P, _P, _P,
+                                   _P]),
+    "tv_lm_head": (_I, [_P, _I, _I, _P, _P, _F, _P, _P, _P]),
     "tv_get_status": (_I, [_P, ctypes.POINTER(ctypes.c_uint32)]),
     "tv_debug_withhold_job": (_I, [_P, _I]),
     "tv_destroy": (_I, [_P]),
@@ -184,6 +187,40 @@ class Verifier:
         if rc != 0:
             raise LibraryError("tv_verify_batch", rc, self.lib)
         return path, tau, bonus
+
+    def lm_head(self, hidden, weight, temperature, stream=None):
+        """Logits [M, V] bf16 = hidden [M, K] x weight [V, K]^T on the tensor
+        cores, and each row's normaliser [M, 2] fp32 (max, sum of
+        2^((l - max) log2(e) / T)) of the stored logits (tv_lm_head)."""
+        import torch
+        M, K = hidden.shape
+        logits = torch.empty(M, self.vocab, dtype=torch.bfloat16, device=self.device)
+        row_stats = torch.empty(M, 2, dtype=torch.float32, device=self.device)
+        rc = self.lib.tv_lm_head(self.handle, M, K, _ptr(hidden), _ptr(weight),
+                                 float(temperature), _ptr(logits), _ptr(row_stats),
+                                 _stream_ptr(stream))
+        if rc != 0:
+            raise LibraryError("tv_lm_head", rc, self.lib)
+        return logits, row_stats
+
+    def verify_stats(self, parents, tokens, logits, drafts, temperature, uniforms, row_stats,
+                     stream=None, debug=False):
+        """verify() with the rows' normalisers given ([B, N+1, 2] or [B*(N+1), 2]
+        fp32, e.g. from lm_head) (tv_verify_batch_stats)."""
+        import torch
+        B, N = self._check(parents, tokens, logits, drafts, uniforms)
+        path = torch.empty(B, N, dtype=torch.int32, device=self.device)
+        tau = torch.empty(B, dtype=torch.int32, device=self.device)
+        bonus = torch.empty(B, dtype=torch.int32, device=self.device)
+        node_p = torch.empty(B, N + 1, dtype=torch.float32, device=self.device) if debug else None
+        stats = torch.empty(B, 5, dtype=torch.int32, device=self.device) if debug else None
+        rc = self.lib.tv_verify_batch_stats(
+            self.handle, B, N, _ptr(parents), _ptr(tokens), _ptr(logits), _ptr(drafts),
+            float(temperature), _ptr(uniforms), _ptr(row_stats), _ptr(path), _ptr(tau),
+            _ptr(bonus), _ptr(node_p), _ptr(stats), _stream_ptr(stream))
+        if rc != 0:
+            raise LibraryError("tv_verify_batch_stats", rc, self.lib)
+        return (path, tau, bonus, node_p, stats) if debug else (path, tau, bonus)
 
     def verify_host(self, parents, tokens, logits, drafts, temperature, uniforms,
                     out, stream=None):

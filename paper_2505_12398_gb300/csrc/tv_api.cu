@@ -34,6 +34,9 @@ struct tv_handle {
   size_t flow_ws_bytes = 0;
   unsigned long long epoch = 0;  // per-call tag of the persistent kernel's queue
   int withhold_tree = -1;        // test hook for the next persistent call (-1: none)
+  // per-(row, tile) scratch of tv_lm_head (allocated on first use)
+  float2* lmh_part = nullptr;
+  size_t lmh_part_bytes = 0;
   // staging for tv_verify_batch_host (allocated on first use)
   char* stage = nullptr;
   size_t stage_bytes = 0;
@@ -114,7 +117,8 @@ int check_call(const tv_handle* h, int B, int N, const void* parents, const void
 int verify_impl(tv_handle* h, int B, int N, const int32_t* parents, const int32_t* tokens,
                 const void* logits, const float* drafts, float temperature,
                 const float* uniforms, int32_t* out_path, int32_t* out_len, int32_t* out_bonus,
-                float* out_node_p, int32_t* out_stats, void* stream) {
+                float* out_node_p, int32_t* out_stats, void* stream,
+                const float2* row_stats = nullptr) {
   int rc = check_call(h, B, N, parents, tokens, logits, drafts, temperature, uniforms,
                       out_path, out_len, out_bonus);
   if (rc != TV_OK || B == 0) return rc;
@@ -141,6 +145,7 @@ int verify_impl(tv_handle* h, int B, int N, const int32_t* parents, const int32_
   a.out_stats = out_stats;
   a.status = h->status;
   a.token_level = (h->flags & TV_FLAG_TOKEN_LEVEL) ? 1 : 0;
+  a.row_stats = row_stats;
   const int rows = B * (N + 1);
   int grid = h->sm_count * 4;
   if (grid > rows) grid = rows;
@@ -149,6 +154,8 @@ int verify_impl(tv_handle* h, int B, int N, const int32_t* parents, const int32_
   const Path path = choose_path(h, B, N + 1, &plan);
   // the three-kernel path implements Traversal Verification only
   if (path == kPathThree && a.token_level) return TV_ERR_INVALID_ARG;
+  // given row normalisers are read by the persistent kernel only
+  if (row_stats && path != kPathPersistent) return TV_ERR_INVALID_ARG;
   const int bf16 = h->dtype == TV_BF16 ? 1 : 0;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   cudaEvent_t* ev = h->timing ? h->ev : nullptr;
@@ -346,6 +353,52 @@ int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
   return TV_OK;
 }
 
+int tv_verify_batch_stats(tv_handle* h, int B, int N, const int32_t* parents,
+                          const int32_t* draft_tokens, const void* target_logits,
+                          const float* draft_probs, float temperature, const float* uniforms,
+                          const float* row_stats, int32_t* out_accepted_path,
+                          int32_t* out_accept_len, int32_t* out_bonus_token, float* out_node_p,
+                          int32_t* out_stats, void* cuda_stream) {
+  if (!row_stats || (reinterpret_cast<uintptr_t>(row_stats) & 7u)) return TV_ERR_INVALID_ARG;
+  return verify_impl(h, B, N, parents, draft_tokens, target_logits, draft_probs, temperature,
+                     uniforms, out_accepted_path, out_accept_len, out_bonus_token, out_node_p,
+                     out_stats, cuda_stream, reinterpret_cast<const float2*>(row_stats));
+}
+
+int tv_lm_head(tv_handle* h, int M, int K, const void* hidden, const void* weight,
+               float temperature, void* out_logits, float* out_row_stats, void* cuda_stream) {
+  if (!h || M < 0 || K < 64 || (K % 64) != 0) return TV_ERR_INVALID_ARG;
+  if (h->dtype != TV_BF16 || (h->vocab % 8) != 0) return TV_ERR_INVALID_ARG;
+  if ((size_t)M > (size_t)h->max_batch * (h->max_nodes + 1)) return TV_ERR_CAPACITY;
+  if (!(std::isfinite(temperature) && temperature > 0.f)) return TV_ERR_TEMPERATURE;
+  if (M == 0) return TV_OK;
+  if (!hidden || !weight || !out_logits || !out_row_stats || !aligned16(hidden) ||
+      !aligned16(weight) || !aligned16(out_logits) ||
+      (reinterpret_cast<uintptr_t>(out_row_stats) & 7u))
+    return TV_ERR_INVALID_ARG;
+  DeviceGuard guard(h->device);
+  if (!guard.ok()) return TV_ERR_CUDA;
+  const size_t need = (size_t)h->max_batch * (h->max_nodes + 1) *
+                      (size_t)tv_lm_head_tiles(h->vocab) * sizeof(float2);
+  if (h->lmh_part_bytes < need) {
+    if (h->lmh_part) cudaFree(h->lmh_part);
+    h->lmh_part = nullptr;
+    h->lmh_part_bytes = 0;
+    if (cudaMalloc(&h->lmh_part, need) != cudaSuccess) {
+      cudaGetLastError();
+      return TV_ERR_CUDA;
+    }
+    h->lmh_part_bytes = need;
+  }
+  const double c = 1.4426950408889634 / static_cast<double>(temperature);
+  const float c_hi = static_cast<float>(c);
+  const float c_lo = static_cast<float>(c - static_cast<double>(c_hi));
+  const int rc = tv_launch_lm_head(hidden, weight, M, K, h->vocab, c_hi, c_lo, out_logits,
+                                   h->lmh_part, reinterpret_cast<float2*>(out_row_stats),
+                                   h->status, static_cast<cudaStream_t>(cuda_stream));
+  return rc == 0 ? TV_OK : TV_ERR_CUDA;
+}
+
 int tv_debug_withhold_job(tv_handle* h, int tree) {
   if (!h || tree < 0 || tree >= h->max_batch) return TV_ERR_INVALID_ARG;
   h->withhold_tree = tree;
@@ -426,6 +479,7 @@ int tv_destroy(tv_handle* h) {
     cudaFree(h->status);
     if (h->flow_ws) cudaFree(h->flow_ws);
     if (h->stage) cudaFree(h->stage);
+    if (h->lmh_part) cudaFree(h->lmh_part);
     cudaGetLastError();
   }
   delete h;

@@ -760,7 +760,7 @@ __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const
 }
 
 // Structure, validation and gathers of tree b; leaves ctl ready to run.
-template <typename L>
+template <typename L, bool kGiven>
 __device__ void owner_new_tree(const TravArgs& a, const TreeSmem& s, Shared& sh, float* u,
                                int b, int lane) {
   const int R = a.N + 1, V = a.V;
@@ -832,6 +832,26 @@ __device__ void owner_new_tree(const TravArgs& a, const TreeSmem& s, Shared& sh,
     bad = __reduce_or_sync(0xffffffffu, bad2);
   }
   __syncwarp();
+  if (kGiven && bad == 0u) {
+    // given normalisers (from the LM head's epilogue): every internal row is
+    // normalised up front and no stats job is ever posted
+    uint32_t bad3 = 0u;
+    for (int i = lane; i < R; i += 32) {
+      if (s.first[i] < 0) continue;
+      const float2 st = a.row_stats[row0 + i];
+      s.rowm[i] = st.x;
+      s.rows[i] = st.y;
+      s.invs[i] = 1.0 / (double)st.y;
+      if (!(st.y > 0.f)) bad3 |= 64u;
+    }
+    __syncwarp();
+    for (int i = lane + 1; i < R; i += 32) {
+      const int p = s.par[i];
+      s.mb0[i] = exp2(((double)s.gl[i] - (double)s.rowm[p]) * a.c) * s.invs[p];
+    }
+    bad = __reduce_or_sync(0xffffffffu, bad3);
+    __syncwarp();
+  }
   if (lane == 0) {
     sh.ctl.bad = bad;
     if (bad == 0u) {
@@ -1061,6 +1081,7 @@ __device__ void owner_combine(const TravArgs& a, const FlowArgs& f, const TreeSm
 }
 
 // Writes tree b's outputs; true if it was the last tree of the call.
+template <bool kGiven>
 __device__ bool owner_finish(const TravArgs& a, const FlowArgs& f, const TreeSmem& s,
                              Shared& sh, int b, int lane) {
   const int R = a.N + 1, N = a.N;
@@ -1094,7 +1115,7 @@ __device__ bool owner_finish(const TravArgs& a, const FlowArgs& f, const TreeSme
       o[1] = ok ? sh.ctl.n_passes : 0;
       o[2] = ok ? distinct : 0;
       o[3] = (acc_node >= 0 && s.first[acc_node] < 0) ? 1 : 0;
-      o[4] = ok ? normalised : 0;
+      o[4] = (ok && !kGiven) ? normalised : 0;   // rows this call streamed
     }
     if (sh.ctl.bad) atomicOr(a.status, sh.ctl.bad);
     f.finished[b] = (unsigned)f.epoch;
@@ -1105,7 +1126,7 @@ __device__ bool owner_finish(const TravArgs& a, const FlowArgs& f, const TreeSme
   return __shfl_sync(0xffffffffu, last, 0) != 0;
 }
 
-template <typename L>
+template <typename L, bool kGiven>
 __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, int lane) {
   const int R = a.N + 1, V = a.V, B = a.B;
   Shared& sh = *m.sh;
@@ -1125,7 +1146,7 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
       t = __shfl_sync(0xffffffffu, t, 0);
       if (t >= (unsigned)B) break;   // no trees left for this CTA to own
       my_tree = (int)t;
-      owner_new_tree<L>(a, s, sh, m.u, my_tree, lane);
+      owner_new_tree<L, kGiven>(a, s, sh, m.u, my_tree, lane);
     } else {
       // poll the own job's partials (kept in pbuf for the combine)
       const int nout = sh.outstanding;
@@ -1240,7 +1261,7 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
     if (sh.ctl.job.kind == kJobDone) {
       if (spec.n > 0) post_nops(a, f, spec, lane);   // before the tree counts as done
       spec.n = 0;
-      const bool last = owner_finish(a, f, s, sh, my_tree, lane);
+      const bool last = owner_finish<kGiven>(a, f, s, sh, my_tree, lane);
       my_tree = -1;
       if (last) {
         // every tree is done: the tickets now held (slots from the tail up to
@@ -1271,7 +1292,10 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
 
 // ------------------------------------------------------------- the kernel --
 
-template <typename L, int kNCW>
+// kGiven: the rows' normalisers come with the call (args.row_stats), so no
+// stats job is ever posted; a separate instantiation keeps the owner code of
+// the common case free of that branch
+template <typename L, int kNCW, bool kGiven>
 __global__ void __launch_bounds__(Shape<L, kNCW>::kThreads, 16 / kNCW)
     tv_flow_kernel(TravArgs args, FlowArgs f, int n_stages) {
   using S = Shape<L, kNCW>;
@@ -1318,7 +1342,7 @@ __global__ void __launch_bounds__(Shape<L, kNCW>::kThreads, 16 / kNCW)
   if (wid < kNCW) consumer_role<L, kNCW>(args, f, m, n_stages, wid, lane);
   else if (wid == kNCW) producer_role<L, kNCW>(args, f, m, n_stages, lane);
   else if (wid == kNCW + 1) fetcher_role<L, kNCW>(args, f, m, lane);
-  else owner_role<L>(args, f, m, lane);
+  else owner_role<L, kGiven>(args, f, m, lane);
 
   // ---------------- exit ----------------
   __syncthreads();
@@ -1443,7 +1467,7 @@ struct LaunchCache {
 };
 constexpr int kCacheDevices = 64;
 std::mutex g_launch_mutex;
-LaunchCache g_launch_cache[kCacheDevices][4];
+LaunchCache g_launch_cache[kCacheDevices][8];
 
 }  // namespace
 
@@ -1496,15 +1520,25 @@ int tv_launch_flow(const TravArgs& a, FlowArgs f, int logit_is_bf16, const FlowP
     }
     return 0;
   };
+  using tvk::Bf16Logits;
+  using tvk::F32Logits;
+  const int given = a.row_stats != nullptr;
   int rc;
-  if (plan.ncw == 8)
-    rc = logit_is_bf16
-             ? run(tv_flow_kernel<tvk::Bf16Logits, 8>, Shape<tvk::Bf16Logits, 8>::kThreads, 0)
-             : run(tv_flow_kernel<tvk::F32Logits, 8>, Shape<tvk::F32Logits, 8>::kThreads, 1);
-  else
-    rc = logit_is_bf16
-             ? run(tv_flow_kernel<tvk::Bf16Logits, 4>, Shape<tvk::Bf16Logits, 4>::kThreads, 2)
-             : run(tv_flow_kernel<tvk::F32Logits, 4>, Shape<tvk::F32Logits, 4>::kThreads, 3);
+  if (plan.ncw == 8) {
+    if (logit_is_bf16)
+      rc = given ? run(tv_flow_kernel<Bf16Logits, 8, true>, Shape<Bf16Logits, 8>::kThreads, 4)
+                 : run(tv_flow_kernel<Bf16Logits, 8, false>, Shape<Bf16Logits, 8>::kThreads, 0);
+    else
+      rc = given ? run(tv_flow_kernel<F32Logits, 8, true>, Shape<F32Logits, 8>::kThreads, 5)
+                 : run(tv_flow_kernel<F32Logits, 8, false>, Shape<F32Logits, 8>::kThreads, 1);
+  } else {
+    if (logit_is_bf16)
+      rc = given ? run(tv_flow_kernel<Bf16Logits, 4, true>, Shape<Bf16Logits, 4>::kThreads, 6)
+                 : run(tv_flow_kernel<Bf16Logits, 4, false>, Shape<Bf16Logits, 4>::kThreads, 2);
+    else
+      rc = given ? run(tv_flow_kernel<F32Logits, 4, true>, Shape<F32Logits, 4>::kThreads, 7)
+                 : run(tv_flow_kernel<F32Logits, 4, false>, Shape<F32Logits, 4>::kThreads, 3);
+  }
   if (rc) return rc;
   if (ev && cudaEventRecord(ev[3], stream) != cudaSuccess) return -5;
   return 0;

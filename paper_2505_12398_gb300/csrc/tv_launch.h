@@ -22,6 +22,8 @@ struct TravArgs {
   int32_t* out_stats;          // [B][4] or nullptr
   uint32_t* status;            // status word (OR of TV_STATUS_* bits)
   int token_level;             // 1: token-level (top-down) verification instead (fused paths)
+  const float2* row_stats;     // [B][N+1] given row normalisers (max, sum), or nullptr
+                               // (persistent path)
 };
 
 // Launch plan of the fused kernel: cluster size, ring stages, shared memory.
@@ -110,3 +112,17 @@ int tv_flow_bind(void* base, size_t bytes, int B, int R, int V, const FlowPlan& 
 // tv_launch_fused.
 int tv_launch_flow(const TravArgs& a, FlowArgs f, int logit_is_bf16, const FlowPlan& plan,
                    int sm_count, cudaStream_t stream, cudaEvent_t* events);
+
+// ---- LM head fused with the row normalisers (tv_gemm.cu) ----
+
+// Tiles of 256 logits per row (the per-row workspace of tv_launch_lm_head).
+int tv_lm_head_tiles(int V);
+// logits[M][V] (bf16) = hidden[M][K] x weight[V][K]^T (bf16) on the tensor
+// cores, and row_stats[M] = (max, sum of 2^((l - max) (c_hi + c_lo))) of the
+// stored logits.  part is [M][tv_lm_head_tiles(V)] scratch.  Requires K % 64
+// == 0, V % 8 == 0 and 16-byte aligned arrays.  0 on success, -5 on a CUDA
+// or tensor-map error.
+int tv_launch_lm_head(const void* hidden, const void* weight, int M, int K, int V, float c_hi,
+                      float c_lo, void* logits, float2* part, float2* row_stats,
+                      uint32_t* status, cudaStream_t stream);
+

@@ -139,6 +139,7 @@ extern "C" int tv_verify_batch_noalloc(int device, int B, int N, int vocab, tv_d
       a.out_stats = nullptr;
       a.status = status;
       a.token_level = 0;
+      a.row_stats = nullptr;
       const int rows = B * (N + 1);
       int grid = g_sm_count[device] * 4;
       if (grid > rows) grid = rows;
