@@ -44,6 +44,12 @@ def parse_args():
                          "(top-down RRS without replacement) verifier it is compared with")
     ap.add_argument("--path", choices=["auto", "persistent", "cluster", "three"], default="auto",
                     help="kernel path of the handle (auto: the library's choice)")
+    ap.add_argument("--pipeline", choices=["verify", "lmhead"], default="verify",
+                    help="verify: one step = one verification call; lmhead: one step = the "
+                         "target LM head (logits and row normalisers on the tensor cores) "
+                         "followed by verification with those normalisers")
+    ap.add_argument("--hidden", type=int, default=4096,
+                    help="hidden size K of the LM head (--pipeline lmhead)")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -81,14 +87,17 @@ def whole_job_rate(units_per_rank, world, repeats, total_ms):
 
 # sources of the persistent kernel, in the order its profile's hash covers them
 FLOW_SOURCES = ["tv_control.cuh", "tv_device.cuh", "tv_flow.cu", "tv_launch.h", "tv_ptx.cuh"]
+GEMM_SOURCES = ["tv_device.cuh", "tv_gemm.cu", "tv_launch.h", "tv_ptx.cuh"]
 
 
-def kernel_traffic(workload, batch):
-    """DRAM bytes per launch of the persistent kernel from the committed ncu
+def kernel_traffic(workload, batch, kind="persistent"):
+    """DRAM bytes per launch of the dominant kernel (kind "persistent": the
+    verification kernel; "lmhead": the LM-head GEMM) from the committed ncu
     summary of this workload, or None when there is none or the kernel's
     sources have changed since it was taken."""
     import hashlib
-    path = os.path.join(ROOT, "profiles", f"launches_{workload}_B{batch}_persistent.md")
+    sources = GEMM_SOURCES if kind == "lmhead" else FLOW_SOURCES
+    path = os.path.join(ROOT, "profiles", f"launches_{workload}_B{batch}_{kind}.md")
     if not os.path.exists(path):
         return None
     fields = {}
@@ -101,7 +110,7 @@ def kernel_traffic(workload, batch):
         return None
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2505_12398_gb300", "csrc")
-    for name in FLOW_SOURCES:
+    for name in sources:
         h.update(name.encode())
         with open(os.path.join(csrc, name), "rb") as f:
             h.update(f.read())
@@ -118,6 +127,18 @@ def measured_peaks():
         return float(d["hbm_gbs"]), "measured"
     except Exception:
         return 6800.0, "fallback"
+
+
+def measured_bf16_peak():
+    """Dense bf16 tensor peak in TFLOP/s: the measured burst figure (a kernel
+    timed on its own) or the fallback."""
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["bf16_tflops"]), "measured"
+    except Exception:
+        return 1900.0, "fallback"
 
 
 # ----------------------------------------------------------- clocks ---------
@@ -253,7 +274,11 @@ def main():
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
 
     if args.impl == "reference":
+        if args.pipeline == "lmhead":
+            return run_reference_lmhead(args, world, rank)
         return run_reference(args, world, rank)
+    if args.pipeline == "lmhead":
+        return main_lmhead(args, world, rank, local_rank)
 
     import torch
     import torch.distributed as dist
@@ -493,6 +518,300 @@ def run_reference(args, world, rank):
                          "kind": "oracle",
                          "sample": f"{per_step} trees of the workload per step, one per "
                                    f"spawn worker"},
+        "e2e": {"value": round(value, 4), "unit": "trees/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------- LM-head pipeline ---------
+
+def dump_lmhead_sample(lin, trees, tmpdir):
+    """Host copies, for the oracle, of the sampled trees' hidden states and
+    draft side, and of the output embedding (bf16 bit patterns)."""
+    import numpy as np
+    import torch
+    inp = lin.inputs
+    idx = list(trees)
+    R = inp.parents.shape[1]
+    outdir = os.path.join(tmpdir, "lmhead")
+    os.makedirs(outdir, exist_ok=True)
+    rows = torch.cat([torch.arange(b * R, (b + 1) * R) for b in idx]).to(lin.hidden.device)
+    arrays = {
+        "hidden": lin.hidden.index_select(0, rows).view(torch.int16).cpu().numpy(),
+        "weight": lin.weight.view(torch.int16).cpu().numpy(),
+        "parents": inp.parents[idx].cpu().numpy(), "tokens": inp.tokens[idx].cpu().numpy(),
+        "drafts": inp.draft_probs[idx].cpu().numpy(), "uniforms": inp.uniforms[idx].cpu().numpy(),
+    }
+    for k, a in arrays.items():
+        np.save(os.path.join(outdir, k + ".npy"), a)
+    return outdir
+
+
+def _bf16_bits_to_f64(a):
+    import numpy as np
+    return (a.astype(np.uint16).astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def _lmhead_oracle_worker(args):
+    """One tree through the oracle: logits of its rows (float64 products,
+    stored as bf16), then Algorithm 3 on them."""
+    path, b, temperature = args
+    import numpy as np
+    from oracle import lmhead
+    from oracle.verify import verify_tree
+    d = _DirArrays(path)
+    R = d["parents"].shape[1]
+    h = _bf16_bits_to_f64(np.asarray(d["hidden"][b * R:(b + 1) * R]))
+    wt = d["weight"]
+    V = wt.shape[0]
+    logits = np.empty((R, V))
+    step = 8192                       # output columns per chunk: bounds the float64 copy of W
+    for v0 in range(0, V, step):
+        v1 = min(V, v0 + step)
+        logits[:, v0:v1] = lmhead.logits(h, _bf16_bits_to_f64(np.asarray(wt[v0:v1])))
+    stored = lmhead.to_bf16(logits)
+    r = verify_tree(d["parents"][b], d["tokens"][b], stored, d["drafts"][b], temperature,
+                    d["uniforms"][b])
+    return r["tau"]
+
+
+def time_lmhead_oracle(sample_dir, n_trees, temperature, pool, reps=1):
+    jobs = [(sample_dir, b % n_trees, temperature) for b in range(n_trees * reps)]
+    t0 = time.perf_counter()
+    taus = pool.map(_lmhead_oracle_worker, jobs, chunksize=1)
+    return time.perf_counter() - t0, len(jobs), taus
+
+
+def _oracle_pool(cores):
+    """A spawn pool whose workers run single-threaded BLAS (one tree each)."""
+    import multiprocessing as mp
+    for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        os.environ[k] = "1"
+    return mp.get_context("spawn").Pool(cores)
+
+
+def main_lmhead(args, world, rank, local_rank):
+    """One step = tv_lm_head (logits and row normalisers of every row of the
+    batch, tensor cores) then tv_verify_batch_stats on them."""
+    import torch
+    import torch.distributed as dist
+    import paper_2505_12398_gb300 as tv
+    from paper_2505_12398_gb300.build import build
+    from workloads.synth import get_workload, make_lmhead_inputs
+
+    if world > 1:
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local_rank if world > 1 else 0)
+    torch.cuda.set_device(dev)
+    build()
+
+    w = get_workload(args.workload, batch=args.batch, sigma=args.sigma,
+                     logit_dtype=torch.bfloat16)
+    lin = make_lmhead_inputs(w, hidden=args.hidden, seed=rank_seed(args.seed, rank), device=dev)
+    inp = lin.inputs
+    B, R = inp.parents.shape
+    N, V, K = R - 1, w.vocab, args.hidden
+    M = B * R
+    v = tv.Verifier(V, N, B, "bf16", device=dev.index, path="persistent", method=args.method)
+    stream = torch.cuda.current_stream(dev)
+    logits = torch.empty(B, R, V, dtype=torch.bfloat16, device=dev)
+    row_stats = torch.empty(M, 2, dtype=torch.float32, device=dev)
+    lm_out = (logits.view(M, V), row_stats)
+    out = (torch.empty(B, N, dtype=torch.int32, device=dev),
+           torch.empty(B, dtype=torch.int32, device=dev),
+           torch.empty(B, dtype=torch.int32, device=dev))
+
+    def step():
+        v.lm_head(lin.hidden, lin.weight, inp.temperature, out=lm_out, stream=stream)
+        v.verify_stats(inp.parents, inp.tokens, logits, inp.draft_probs, inp.temperature,
+                       inp.uniforms, row_stats, out=out, stream=stream)
+
+    # instrumented call: the rows each tree reads, tau
+    v.lm_head(lin.hidden, lin.weight, inp.temperature, out=lm_out, stream=stream)
+    _, tau_d, _, _, stats = v.verify_stats(inp.parents, inp.tokens, logits, inp.draft_probs,
+                                           inp.temperature, inp.uniforms, row_stats,
+                                           stream=stream, debug=True)
+    torch.cuda.synchronize(dev)
+    if v.status() & ~16:
+        raise RuntimeError(f"device status {tv.status_names(v.status())}")
+    _, trav_bytes = algorithmic_bytes(stats, tau_d, V, 2)
+    mean_tau1 = float(tau_d.float().mean()) + 1.0
+
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    for _ in range(args.warmup):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize(dev)
+
+    gpu_idx = 0
+    cvd = os.environ.get("CUDA_VISIBLE_DEVICES", "")
+    if cvd and cvd.split(",")[dev.index].strip().isdigit():
+        gpu_idx = int(cvd.split(",")[dev.index])
+    sampler = ClockSampler(gpu_idx)
+    sampler.start()
+    time.sleep(0.3)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    wall0 = time.perf_counter()
+    for k in range(args.steps):
+        flush.zero_()
+        ev[k][0].record(stream)
+        v.lm_head(lin.hidden, lin.weight, inp.temperature, out=lm_out, stream=stream)
+        ev[k][1].record(stream)
+        v.verify_stats(inp.parents, inp.tokens, logits, inp.draft_probs, inp.temperature,
+                       inp.uniforms, row_stats, out=out, stream=stream)
+        ev[k][2].record(stream)
+    torch.cuda.synchronize(dev)
+    wall = time.perf_counter() - wall0
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop()
+    gemm_ms = sum(e[0].elapsed_time(e[1]) for e in ev) / args.steps
+    ver_ms = sum(e[1].elapsed_time(e[2]) for e in ev) / args.steps
+    total_ms = sum(e[0].elapsed_time(e[2]) for e in ev)
+    total_ms_max = max_over_ranks(total_ms, world, dev)
+
+    # end to end: hidden states and the draft side from pinned host memory,
+    # outputs back to the host, every step
+    e2e = None
+    if not args.no_e2e:
+        hp = [x.cpu().pin_memory() for x in (lin.hidden, inp.parents, inp.tokens,
+                                              inp.draft_probs, inp.uniforms)]
+        dbuf = [torch.empty_like(x, device=dev) for x in hp]
+        hout = [torch.empty(o.shape, dtype=o.dtype).pin_memory() for o in out]
+
+        def e2e_step():
+            for d, h in zip(dbuf, hp):
+                d.copy_(h, non_blocking=True)
+            v.lm_head(dbuf[0], lin.weight, inp.temperature, out=lm_out, stream=stream)
+            v.verify_stats(dbuf[1], dbuf[2], logits, dbuf[3], inp.temperature, dbuf[4],
+                           row_stats, out=out, stream=stream)
+            for h, o in zip(hout, out):
+                h.copy_(o, non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize(dev)
+        ks = max(1, args.e2e_steps)
+        if world > 1:
+            dist.barrier()
+        x0 = torch.cuda.Event(enable_timing=True)
+        x1 = torch.cuda.Event(enable_timing=True)
+        x0.record(stream)
+        for _ in range(ks):
+            e2e_step()
+        x1.record(stream)
+        torch.cuda.synchronize(dev)
+        e_ms_max = max_over_ranks(x0.elapsed_time(x1), world, dev)
+        assert torch.equal(hout[1], out[1].cpu()), "end-to-end outputs disagree"
+        e2e = {"value": round(whole_job_rate(B, world, ks, e_ms_max), 3), "unit": "trees/s",
+               "h2d_bytes_per_step": int(sum(x.numel() * x.element_size() for x in hp)),
+               "d2h_bytes_per_step": int(sum(x.numel() * x.element_size() for x in hout)),
+               "steps": ks}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline_lmhead(lin, args, B)
+
+    peak, peak_kind = measured_bf16_peak()
+    hbm, hbm_kind = measured_peaks()
+    flops = 2.0 * M * K * V
+    gemm_tflops = flops / (gemm_ms / 1e3) / 1e12
+    ver_gbs = trav_bytes / (ver_ms / 1e3) / 1e9
+    ms_step = total_ms_max / args.steps
+    line = {
+        "metric": "verified trees/sec including the target LM head (logits + row "
+                  "normalisers on the tensor cores, then verification), 1 GB300",
+        "value": round(whole_job_rate(B, world, args.steps, total_ms_max), 3),
+        "unit": "trees/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(ms_step, 6), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (hidden states and output embedding whose product has the "
+                "workload's logit law; draft side drawn from those logits)",
+        "config": {"workload": w.name, "pipeline": "lmhead", "batch": B, "vocab": V,
+                   "nodes": N, "hidden": K, "rows": M, "method": args.method,
+                   "temperature": w.temperature, "sigma": w.sigma, "seed": args.seed,
+                   "l2": "flushed by a 256 MiB write before every timed step (untimed)",
+                   "parallelism": f"dp{world} (independent trees per GPU)"},
+        "phase_ms": {"lm_head_kernel+lm_head_merge_kernel": round(gemm_ms, 6),
+                     "tv_flow_kernel (given normalisers)": round(ver_ms, 6)},
+        "mean_accept_len_tau_plus_1": round(mean_tau1, 4),
+        "roofline": {"bound": "tensor", "kernel": "lm_head_kernel",
+                     "achieved": round(gemm_tflops, 2), "peak": peak, "unit": "TFLOP/s",
+                     "frac": round(gemm_tflops / peak, 4), "peak_kind": peak_kind + " (burst)",
+                     "flops_per_launch": flops,
+                     "traffic": kernel_traffic(w.name, B, "lmhead")},
+        "roofline_verify": {"bound": "hbm", "kernel": "tv_flow_kernel",
+                            "achieved": round(ver_gbs, 2), "peak": hbm, "unit": "GB/s",
+                            "frac": round(ver_gbs / hbm, 4), "peak_kind": hbm_kind,
+                            "bytes_per_launch": trav_bytes},
+        "e2e": e2e,
+        "gpu_launches": 3 * args.steps,
+        "clocks": clocks,
+        "cpu_baseline": cpu,
+        "wall_s_timed_region": round(wall, 3),
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    v.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def cpu_baseline_lmhead(lin, args, B):
+    cores = os.cpu_count() or 1
+    with tempfile.TemporaryDirectory() as td:
+        n_sample = min(B, cores)
+        sdir = dump_lmhead_sample(lin, range(n_sample), td)
+        with _oracle_pool(cores) as pool:
+            t_probe, _, _ = time_lmhead_oracle(sdir, n_sample, lin.inputs.temperature, pool)
+            reps = max(1, min(50, int(args.cpu_seconds / max(t_probe, 1e-3))))
+            t, n, _ = time_lmhead_oracle(sdir, n_sample, lin.inputs.temperature, pool, reps=reps)
+    return {"value": round(n / t, 4), "unit": "trees/s", "cores": cores, "kind": "oracle",
+            "sample": f"{n} trees ({n_sample} distinct trees of the batch, repeated {reps}x) "
+                      f"through the oracle LM head (float64 products, bf16 storage) and "
+                      f"verification, one tree per single-threaded spawn worker, {t:.1f} s"}
+
+
+def run_reference_lmhead(args, world, rank):
+    """The oracle LM head and verification as the reference arm."""
+    if rank != 0:
+        return
+    import torch
+    from workloads.synth import get_workload, make_lmhead_inputs
+    w = get_workload(args.workload, batch=args.batch, sigma=args.sigma)
+    cores = os.cpu_count() or 1
+    per_step = max(1, min(w.batch, cores))
+    gen_w = get_workload(args.workload, batch=per_step, sigma=args.sigma,
+                         logit_dtype=torch.bfloat16)
+    lin = make_lmhead_inputs(gen_w, hidden=args.hidden, seed=args.seed, device="cpu")
+    with tempfile.TemporaryDirectory() as td:
+        sdir = dump_lmhead_sample(lin, range(per_step), td)
+        with _oracle_pool(cores) as pool:
+            for _ in range(args.warmup):
+                time_lmhead_oracle(sdir, per_step, lin.inputs.temperature, pool)
+            times = [time_lmhead_oracle(sdir, per_step, lin.inputs.temperature, pool)[0]
+                     for _ in range(args.steps)]
+    total = sum(times)
+    value = per_step * args.steps / total
+    line = {
+        "impl": "reference",
+        "metric": "verified trees/sec including the target LM head (logits + row "
+                  "normalisers on the tensor cores, then verification), 1 GB300",
+        "value": round(value, 4), "unit": "trees/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(total / args.steps * 1e3, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": w.name, "pipeline": "lmhead", "batch": w.batch,
+                   "vocab": w.vocab, "nodes": w.nodes, "hidden": args.hidden,
+                   "method": args.method},
+        "cpu_baseline": {"value": round(value, 4), "unit": "trees/s", "cores": cores,
+                         "kind": "oracle",
+                         "sample": f"{per_step} trees of the workload per step, one per "
+                                   f"single-threaded spawn worker"},
         "e2e": {"value": round(value, 4), "unit": "trees/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }

@@ -188,14 +188,22 @@ class Verifier:
             raise LibraryError("tv_verify_batch", rc, self.lib)
         return path, tau, bonus
 
-    def lm_head(self, hidden, weight, temperature, stream=None):
+    def lm_head(self, hidden, weight, temperature, out=None, stream=None):
         """Logits [M, V] bf16 = hidden [M, K] x weight [V, K]^T on the tensor
         cores, and each row's normaliser [M, 2] fp32 (max, sum of
-        2^((l - max) log2(e) / T)) of the stored logits (tv_lm_head)."""
+        2^((l - max) log2(e) / T)) of the stored logits (tv_lm_head).
+        ``out`` = (logits, row_stats) to write into given tensors."""
         import torch
         M, K = hidden.shape
-        logits = torch.empty(M, self.vocab, dtype=torch.bfloat16, device=self.device)
-        row_stats = torch.empty(M, 2, dtype=torch.float32, device=self.device)
+        for t, shape in ((hidden, (M, K)), (weight, (self.vocab, K))):
+            if t.dtype != torch.bfloat16 or tuple(t.shape) != shape or not t.is_contiguous() \
+                    or t.device != self.device:
+                raise ValueError(f"expected a contiguous bf16 {shape} tensor on {self.device}")
+        if out is None:
+            logits = torch.empty(M, self.vocab, dtype=torch.bfloat16, device=self.device)
+            row_stats = torch.empty(M, 2, dtype=torch.float32, device=self.device)
+        else:
+            logits, row_stats = out
         rc = self.lib.tv_lm_head(self.handle, M, K, _ptr(hidden), _ptr(weight),
                                  float(temperature), _ptr(logits), _ptr(row_stats),
                                  _stream_ptr(stream))
@@ -204,14 +212,21 @@ class Verifier:
         return logits, row_stats
 
     def verify_stats(self, parents, tokens, logits, drafts, temperature, uniforms, row_stats,
-                     stream=None, debug=False):
+                     out=None, stream=None, debug=False):
         """verify() with the rows' normalisers given ([B, N+1, 2] or [B*(N+1), 2]
         fp32, e.g. from lm_head) (tv_verify_batch_stats)."""
         import torch
         B, N = self._check(parents, tokens, logits, drafts, uniforms)
-        path = torch.empty(B, N, dtype=torch.int32, device=self.device)
-        tau = torch.empty(B, dtype=torch.int32, device=self.device)
-        bonus = torch.empty(B, dtype=torch.int32, device=self.device)
+        if row_stats.dtype != torch.float32 or row_stats.numel() != 2 * B * (N + 1) or \
+                not row_stats.is_contiguous() or row_stats.device != self.device:
+            raise ValueError("row_stats must be a contiguous float32 [B*(N+1), 2] tensor "
+                             "on the handle's device")
+        if out is None:
+            path = torch.empty(B, N, dtype=torch.int32, device=self.device)
+            tau = torch.empty(B, dtype=torch.int32, device=self.device)
+            bonus = torch.empty(B, dtype=torch.int32, device=self.device)
+        else:
+            path, tau, bonus = out
         node_p = torch.empty(B, N + 1, dtype=torch.float32, device=self.device) if debug else None
         stats = torch.empty(B, 5, dtype=torch.int32, device=self.device) if debug else None
         rc = self.lib.tv_verify_batch_stats(

@@ -10,9 +10,10 @@
 // it stores.  Given those, verification never streams a row for its
 // normaliser.
 //
-// A persistent kernel, one CTA per SM, walks 128 x 256 tiles of l in the
-// order (row tile fastest, then column tile), so that the CTAs running at the
-// same time share W tiles through L2 and W is read from HBM about once:
+// A persistent kernel, one CTA per SM, walks 128 x 256 tiles of l in groups
+// of row tiles holding 32 MiB of H, row tile fastest inside a group, so that
+// the CTAs running at the same time share W tiles through L2 while the
+// group's H stays resident: W is read from HBM once per group, H once.
 //   * warp 0 (one lane) streams 128 x 64 tiles of H and 256 x 64 tiles of W
 //     into a 4-stage shared-memory ring with 2-D TMA copies (128-byte
 //     swizzle, the layout the tensor cores read), across tile boundaries;
@@ -49,6 +50,11 @@ constexpr int kBN = 256;          // columns of a tile (TMEM columns)
 constexpr int kBK = 64;           // K per stage: 128 bytes of bf16, one swizzle row
 constexpr int kUmmaK = 16;        // K per tcgen05.mma of kind::f16
 constexpr int kStages = 4;
+// Tile order: groups of row tiles holding about kGroupBytes of H, row tile
+// fastest inside a group, so that the CTAs running at once share W tiles
+// through L2 while the group's rows of H stay resident.  W is then read from
+// HBM once per group and H once.
+constexpr size_t kGroupBytes = 32u << 20;
 constexpr int kThreads = 192;     // TMA warp, MMA warp, four epilogue warps
 constexpr uint32_t kABytes = kBM * kBK * 2;   // 16 KB
 constexpr uint32_t kBBytes = kBN * kBK * 2;   // 32 KB
@@ -85,6 +91,22 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
       " [%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(dst)),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
       : "memory");
+}
+
+// Row and column tile of the t-th tile in the kernel's order.
+__device__ __forceinline__ void tile_coords(int t, int m_tiles, int n_tiles, int group,
+                                            int& mt, int& nt) {
+  const int g = group > 0 && group < m_tiles ? group : m_tiles;
+  const int full = (m_tiles / g) * g * n_tiles;       // tiles in whole groups
+  if (t < full) {
+    const int grp = t / (g * n_tiles), r = t - grp * g * n_tiles;
+    mt = grp * g + r % g;
+    nt = r / g;
+  } else {
+    const int gt = m_tiles - (m_tiles / g) * g, r = t - full;
+    mt = (m_tiles / g) * g + r % gt;
+    nt = r / gt;
+  }
 }
 
 __device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t a, uint64_t b,
@@ -138,14 +160,14 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-// Tiles t = blockIdx.x, blockIdx.x + gridDim.x, ... of l = H W^T (row tile
-// t % m_tiles, column tile t / m_tiles), stored as bf16, and each row's
+// Tiles t = blockIdx.x, blockIdx.x + gridDim.x, ... of l = H W^T (in the
+// order of tile_coords), stored as bf16, and each row's
 // (max, sum of 2^((l - max) c)) over a tile's columns in part[row][tile].
 __global__ void __launch_bounds__(kThreads, 1)
     lm_head_kernel(const __grid_constant__ CUtensorMap map_h,
                    const __grid_constant__ CUtensorMap map_w, int M, int V, int K, float c_hi,
                    float c_lo, __nv_bfloat16* __restrict__ logits, float2* __restrict__ part,
-                   int m_tiles, int n_tiles, uint32_t* __restrict__ status) {
+                   int m_tiles, int n_tiles, int group, uint32_t* __restrict__ status) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[kStages];
   __shared__ __align__(8) uint64_t empty_bar[kStages];
@@ -186,7 +208,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t it = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < n_total && ok; t += gridDim.x) {
-        const int m0 = (t % m_tiles) * kBM, n0 = (t / m_tiles) * kBN;
+        int mt, nt;
+        tile_coords(t, m_tiles, n_tiles, group, mt, nt);
+        const int m0 = mt * kBM, n0 = nt * kBN;
         for (int kb = 0; kb < nkb; ++kb, ++it) {
           const uint32_t s = it % kStages;
           if (it >= kStages && !mbar_wait(&empty_bar[s], ((it / kStages) - 1) & 1)) {
@@ -255,7 +279,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         break;
       }
       tc_fence_after();
-      const int m0 = (t % m_tiles) * kBM, n_tile = t / m_tiles, n0 = n_tile * kBN;
+      int mt, n_tile;
+      tile_coords(t, m_tiles, n_tiles, group, mt, n_tile);
+      const int m0 = mt * kBM, n0 = n_tile * kBN;
       const int row = m0 + q * 32 + lane;
       const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + acc * (uint32_t)kBN;
       float m_run = TV_NEG_INF, s_run = 0.f;
@@ -421,9 +447,10 @@ int tv_launch_lm_head(const void* hidden, const void* weight, int M, int K, int 
   const int m_tiles = (M + kBM - 1) / kBM;
   // one CTA per SM (its shared memory and all of tensor memory)
   const int grid = std::min(m_tiles * n_tiles, g_gemm_sms[device]);
+  const int group = (int)std::max<size_t>(1, kGroupBytes / ((size_t)kBM * K * 2));
   lm_head_kernel<<<grid, kThreads, kSmemBytes, stream>>>(
       map_h, map_w, M, V, K, c_hi, c_lo, static_cast<__nv_bfloat16*>(logits), part, m_tiles,
-      n_tiles, status);
+      n_tiles, group, status);
   const int warps_per_block = 8;
   lm_head_merge_kernel<<<(M + warps_per_block - 1) / warps_per_block, 32 * warps_per_block, 0,
                          stream>>>(part, M, n_tiles, c_hi, c_lo, row_stats);

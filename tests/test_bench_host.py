@@ -47,3 +47,31 @@ def test_kernel_traffic_follows_the_source_hash(tmp_path, monkeypatch):
     src = root / "paper_2505_12398_gb300" / "csrc" / "tv_flow.cu"
     src.write_text(src.read_text() + "\n// changed\n")
     assert bench.kernel_traffic("eagle_v128k", 128) is None
+
+
+def test_lmhead_oracle_leg_matches_the_oracle_on_the_generated_logits(tmp_path):
+    """The CPU leg of the LM-head pipeline (oracle logits from the dumped
+    bf16 operands, then Algorithm 3) reaches the tau the oracle gives on the
+    generator's own logits (exact operands here, so both hold the same
+    logits)."""
+    import numpy as np
+    from oracle.verify import verify_tree
+    from workloads.synth import get_workload, make_lmhead_inputs
+    w = get_workload("binary4", batch=3, vocab=1024, logit_dtype=torch.bfloat16)
+    lin = make_lmhead_inputs(w, hidden=64, seed=4)
+    # operands k/16 and a bias column of integers: every product is exact
+    g = torch.Generator().manual_seed(9)
+    lin.hidden.copy_((torch.randint(-8, 9, lin.hidden.shape, generator=g) / 16.0).to(torch.bfloat16))
+    lin.weight.copy_((torch.randint(-8, 9, lin.weight.shape, generator=g) / 16.0).to(torch.bfloat16))
+    inp = lin.inputs
+    B, R = inp.parents.shape
+    inp.logits.copy_((lin.hidden.float() @ lin.weight.float().T).view(B, R, -1).to(torch.bfloat16))
+    d = bench.dump_lmhead_sample(lin, range(B), str(tmp_path))
+    with bench._oracle_pool(2) as pool:
+        _, n, taus = bench.time_lmhead_oracle(d, B, inp.temperature, pool)
+    assert n == B
+    for b in range(B):
+        r = verify_tree(inp.parents[b].numpy(), inp.tokens[b].numpy(),
+                        inp.logits[b].float().numpy().astype(np.float64),
+                        inp.draft_probs[b].numpy(), inp.temperature, inp.uniforms[b].numpy())
+        assert taus[b] == r["tau"]

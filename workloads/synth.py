@@ -27,7 +27,13 @@ Recipe (all draws seeded, on any torch device):
   replacement, in child-index order (Definition 1), by Gumbel-top-k on
   log q (the sorted top-k of log q + Gumbel noise is distributed as
   sequential sampling without replacement);
-* uniforms [B, N+2] ~ U[0, 1) float32.
+* uniforms [B, N+2] ~ U[0, 1) float32;
+* for the LM-head pipeline (make_lmhead_inputs): hidden states H [B (N+1), K]
+  and an output embedding W [V, K], bf16, with H[:, 0] = 1 and
+  W[v, 0] = -1.1 ln(1 + pi(v)) (the same rank prior, as a bias column) and
+  the rest N(0, 1) and N(0, 9 / (K - 1)), so l = H W^T has the same law as
+  the logits above up to bf16 rounding of the operands; the draft side is
+  drawn from those logits as above.
 """
 
 from dataclasses import dataclass, field
@@ -228,3 +234,82 @@ def make_inputs_random_shapes(batch, nodes, vocab, seed=0, device="cpu",
     inp.tokens = tokens.to(torch.int32).contiguous()
     inp.meta = {"workload": f"random_shapes_n{nodes}", "seed": seed}
     return inp
+
+
+@dataclass
+class LmHeadInputs:
+    hidden: torch.Tensor        # [B*(N+1), K] bf16
+    weight: torch.Tensor        # [V, K] bf16
+    inputs: Inputs              # tree, tokens, draft probs, uniforms; logits = bf16(H W^T)
+
+
+def make_lmhead_inputs(w: Workload, hidden: int = 4096, seed: int = 0, device="cpu",
+                       chunk_rows: int = 1 << 14):
+    """Hidden states and output embedding whose product is the workload's
+    target logits (see the module docstring), plus the draft side drawn from
+    those logits.  ``inputs.logits`` holds bf16(H W^T) computed here."""
+    dev = torch.device(device)
+    parents = w.tree()
+    n = len(parents)
+    B, V, K = w.batch, w.vocab, hidden
+    g = torch.Generator(device=dev).manual_seed(seed)
+    perm = torch.randperm(V, generator=g, device=dev)
+    H = torch.randn(B * n, K, generator=g, device=dev)
+    H[:, 0] = 1.0
+    H = H.to(torch.bfloat16)
+    W = torch.empty(V, K, dtype=torch.bfloat16, device=dev)
+    scale = 3.0 / float(K - 1) ** 0.5
+    step = max(1, (chunk_rows * 1024) // K)
+    for v0 in range(0, V, step):
+        v1 = min(V, v0 + step)
+        blk = torch.randn(v1 - v0, K, generator=g, device=dev) * scale
+        blk[:, 0] = -1.1 * torch.log1p(perm[v0:v1].to(torch.float32))
+        W[v0:v1] = blk.to(torch.bfloat16)
+        del blk
+    logits = torch.empty(B, n, V, dtype=torch.bfloat16, device=dev)
+    lf = logits.view(B * n, V)
+    rstep = max(1, (chunk_rows * 1024) // V)
+    for r0 in range(0, B * n, rstep):
+        r1 = min(B * n, r0 + rstep)
+        lf[r0:r1] = (H[r0:r1].float() @ W.float().T if dev.type == "cpu"
+                     else H[r0:r1] @ W.T).to(torch.bfloat16)
+    inp = _draft_side(w, parents, logits, seed, dev, chunk_rows)
+    return LmHeadInputs(H.contiguous(), W.contiguous(), inp)
+
+
+def _draft_side(w, parents, logits, seed, dev, chunk_rows):
+    """Draft probabilities, children and uniforms for given target logits
+    (the same recipe as make_inputs)."""
+    n = len(parents)
+    B, V = w.batch, w.vocab
+    g = torch.Generator(device=dev).manual_seed(seed + 500)
+    drafts = torch.empty(B, n, V, dtype=torch.float32, device=dev)
+    lf = logits.view(B * n, V)
+    df = drafts.view(B * n, V)
+    step = max(1, min(B * n, chunk_rows * 1024 // max(V, 1)))
+    inv_t = 1.0 / float(w.temperature)
+    for r0 in range(0, B * n, step):
+        r1 = min(B * n, r0 + step)
+        noise = torch.randn(r1 - r0, V, generator=g, device=dev)
+        df[r0:r1] = torch.softmax((lf[r0:r1].to(torch.float32) + w.sigma * noise) * inv_t,
+                                  dim=-1)
+        del noise
+    gk = torch.Generator(device=dev).manual_seed(seed + 1000)
+    tokens = torch.zeros(B, n, dtype=torch.int64, device=dev)
+    kids = [[] for _ in range(n)]
+    for i in range(1, n):
+        kids[parents[i]].append(i)
+    for i in range(n):
+        if not kids[i]:
+            continue
+        u = torch.rand(B, V, generator=gk, device=dev).clamp_(min=1e-12)
+        keys = torch.log(drafts[:, i, :].clamp(min=1e-38)) - torch.log(-torch.log(u))
+        tokens[:, kids[i]] = torch.topk(keys, len(kids[i]), dim=-1, sorted=True).indices
+        del u, keys
+    gu = torch.Generator(device=dev).manual_seed(seed + 2000)
+    uniforms = torch.rand(B, n + 1, generator=gu, device=dev)
+    uniforms[:, 0] = 0.0
+    par = torch.tensor(parents, dtype=torch.int32, device=dev).expand(B, n).contiguous()
+    return Inputs(par, tokens.to(torch.int32).contiguous(), logits, drafts,
+                  uniforms.contiguous(), float(w.temperature),
+                  {"workload": w.name, "seed": seed, "pipeline": "lmhead"})
