@@ -44,10 +44,11 @@ def parse_args():
                          "(top-down RRS without replacement) verifier it is compared with")
     ap.add_argument("--path", choices=["auto", "persistent", "cluster", "three"], default="auto",
                     help="kernel path of the handle (auto: the library's choice)")
-    ap.add_argument("--pipeline", choices=["verify", "lmhead"], default="verify",
+    ap.add_argument("--pipeline", choices=["verify", "lmhead", "draft"], default="verify",
                     help="verify: one step = one verification call; lmhead: one step = the "
                          "target LM head (logits and row normalisers on the tensor cores) "
-                         "followed by verification with those normalisers")
+                         "followed by verification with those normalisers; draft: one step = "
+                         "drafting every node's children without replacement")
     ap.add_argument("--hidden", type=int, default=4096,
                     help="hidden size K of the LM head (--pipeline lmhead)")
     ap.add_argument("--e2e-steps", type=int, default=10)
@@ -87,7 +88,8 @@ def whole_job_rate(units_per_rank, world, repeats, total_ms):
 
 # sources of the persistent kernel, in the order its profile's hash covers them
 FLOW_SOURCES = ["tv_control.cuh", "tv_device.cuh", "tv_flow.cu", "tv_launch.h", "tv_ptx.cuh"]
-GEMM_SOURCES = ["tv_device.cuh", "tv_gemm.cu", "tv_launch.h", "tv_ptx.cuh"]
+GEMM_SOURCES = ["tv_device.cuh", "tv_gemm.cu", "tv_ptx.cuh"]
+DRAFT_SOURCES = ["tv_draft.cu"]
 
 
 def kernel_traffic(workload, batch, kind="persistent"):
@@ -96,7 +98,7 @@ def kernel_traffic(workload, batch, kind="persistent"):
     summary of this workload, or None when there is none or the kernel's
     sources have changed since it was taken."""
     import hashlib
-    sources = GEMM_SOURCES if kind == "lmhead" else FLOW_SOURCES
+    sources = {"lmhead": GEMM_SOURCES, "draft": DRAFT_SOURCES}.get(kind, FLOW_SOURCES)
     path = os.path.join(ROOT, "profiles", f"launches_{workload}_B{batch}_{kind}.md")
     if not os.path.exists(path):
         return None
@@ -276,9 +278,13 @@ def main():
     if args.impl == "reference":
         if args.pipeline == "lmhead":
             return run_reference_lmhead(args, world, rank)
+        if args.pipeline == "draft":
+            return run_reference_draft(args, world, rank)
         return run_reference(args, world, rank)
     if args.pipeline == "lmhead":
         return main_lmhead(args, world, rank, local_rank)
+    if args.pipeline == "draft":
+        return main_draft(args, world, rank, local_rank)
 
     import torch
     import torch.distributed as dist
@@ -816,6 +822,206 @@ def run_reference_lmhead(args, world, rank):
                 "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------- drafting ---------
+
+def _draft_oracle_worker(args):
+    path, b = args
+    from oracle.drafting import sample_tree
+    d = _DirArrays(path)
+    return sample_tree(d["parents"][b], d["drafts"][b], [float(x) for x in d["uniforms"][b]])
+
+
+def main_draft(args, world, rank, local_rank):
+    """One step = tv_draft_children over the batch: every node's token drawn
+    from its parent's draft row without its earlier siblings' tokens."""
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+    import paper_2505_12398_gb300 as tv
+    from paper_2505_12398_gb300.build import build
+    from workloads.synth import get_workload, internal_rows, make_inputs
+
+    if world > 1:
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local_rank if world > 1 else 0)
+    torch.cuda.set_device(dev)
+    build()
+    w = get_workload(args.workload, batch=args.batch, sigma=args.sigma)
+    inp = make_inputs(w, seed=rank_seed(args.seed, rank), device=dev)
+    B, R = inp.parents.shape
+    N, V = R - 1, w.vocab
+    g = torch.Generator(device=dev).manual_seed(rank_seed(args.seed, rank) + 3000)
+    u = torch.rand(B, R, generator=g, device=dev)
+    v = tv.Verifier(V, N, B, "bf16", device=dev.index, path="three")
+    stream = torch.cuda.current_stream(dev)
+    out = torch.empty(B, R, dtype=torch.int32, device=dev)
+    n_int = len(internal_rows(w.tree()))
+    a_bytes = B * n_int * V * 4 + B * R * 12      # internal draft rows once; parents, u, tokens
+
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    for _ in range(args.warmup):
+        flush.zero_()
+        v.draft_children(inp.parents, inp.draft_probs, u, out=out, stream=stream)
+    torch.cuda.synchronize(dev)
+    if v.status():
+        raise RuntimeError(f"device status {tv.status_names(v.status())}")
+    gpu_idx = 0
+    cvd = os.environ.get("CUDA_VISIBLE_DEVICES", "")
+    if cvd and cvd.split(",")[dev.index].strip().isdigit():
+        gpu_idx = int(cvd.split(",")[dev.index])
+    sampler = ClockSampler(gpu_idx)
+    sampler.start()
+    time.sleep(0.3)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+    wall0 = time.perf_counter()
+    for k in range(args.steps):
+        flush.zero_()
+        ev[k][0].record(stream)
+        v.draft_children(inp.parents, inp.draft_probs, u, out=out, stream=stream)
+        ev[k][1].record(stream)
+    torch.cuda.synchronize(dev)
+    wall = time.perf_counter() - wall0
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop()
+    total_ms = sum(e[0].elapsed_time(e[1]) for e in ev)
+    total_ms_max = max_over_ranks(total_ms, world, dev)
+
+    e2e = None
+    if not args.no_e2e:
+        hp = [x.cpu().pin_memory() for x in (inp.parents, inp.draft_probs, u)]
+        dbuf = [torch.empty_like(x, device=dev) for x in hp]
+        hout = torch.empty(B, R, dtype=torch.int32).pin_memory()
+
+        def e2e_step():
+            for d, h in zip(dbuf, hp):
+                d.copy_(h, non_blocking=True)
+            v.draft_children(dbuf[0], dbuf[1], dbuf[2], out=out, stream=stream)
+            hout.copy_(out, non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize(dev)
+        ks = max(1, args.e2e_steps)
+        if world > 1:
+            dist.barrier()
+        x0 = torch.cuda.Event(enable_timing=True)
+        x1 = torch.cuda.Event(enable_timing=True)
+        x0.record(stream)
+        for _ in range(ks):
+            e2e_step()
+        x1.record(stream)
+        torch.cuda.synchronize(dev)
+        e_ms_max = max_over_ranks(x0.elapsed_time(x1), world, dev)
+        assert torch.equal(hout, out.cpu()), "end-to-end tokens disagree"
+        e2e = {"value": round(whole_job_rate(B, world, ks, e_ms_max), 3), "unit": "trees/s",
+               "h2d_bytes_per_step": int(sum(x.numel() * x.element_size() for x in hp)),
+               "d2h_bytes_per_step": int(hout.numel() * hout.element_size()), "steps": ks}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cores = os.cpu_count() or 1
+        n_sample = min(B, max(cores, 8))
+        with tempfile.TemporaryDirectory() as td:
+            sdir = os.path.join(td, "draft")
+            os.makedirs(sdir)
+            for k, a in (("parents", inp.parents[:n_sample]), ("drafts", inp.draft_probs[:n_sample]),
+                         ("uniforms", u[:n_sample])):
+                np.save(os.path.join(sdir, k + ".npy"), a.cpu().numpy())
+            with _oracle_pool(cores) as pool:
+                jobs = [(sdir, b) for b in range(n_sample)]
+                t0 = time.perf_counter()
+                pool.map(_draft_oracle_worker, jobs, chunksize=1)
+                t_probe = time.perf_counter() - t0
+                reps = max(1, min(200, int(args.cpu_seconds / max(t_probe, 1e-3))))
+                t0 = time.perf_counter()
+                pool.map(_draft_oracle_worker, jobs * reps, chunksize=1)
+                t = time.perf_counter() - t0
+        n = n_sample * reps
+        cpu = {"value": round(n / t, 4), "unit": "trees/s", "cores": cores, "kind": "oracle",
+               "sample": f"{n} trees ({n_sample} distinct trees of the batch, repeated {reps}x) "
+                         f"drafted by the oracle, one tree per single-threaded spawn worker, "
+                         f"{t:.1f} s"}
+
+    peak, peak_kind = measured_peaks()
+    ms_step = total_ms_max / args.steps
+    gbs = a_bytes / (ms_step / 1e3) / 1e9
+    line = {
+        "metric": "drafted trees/sec (every node's children drawn without replacement from "
+                  "its draft row, Definition 1) and draft-row GB/s, 1 GB300",
+        "value": round(whole_job_rate(B, world, args.steps, total_ms_max), 3),
+        "unit": "trees/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(ms_step, 6), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (noisy-drafter probabilities of the workload, uniforms U[0,1))",
+        "config": {"workload": w.name, "pipeline": "draft", "batch": B, "vocab": V, "nodes": N,
+                   "internal_rows_per_tree": n_int, "seed": args.seed,
+                   "l2": "flushed by a 256 MiB write before every timed step (untimed)",
+                   "parallelism": f"dp{world} (independent trees per GPU)"},
+        "roofline": {"bound": "hbm", "kernel": "tv_draft_kernel", "achieved": round(gbs, 2),
+                     "peak": peak, "unit": "GB/s", "frac": round(gbs / peak, 4),
+                     "peak_kind": peak_kind, "bytes_per_launch": a_bytes,
+                     "traffic": kernel_traffic(w.name, B, "draft")},
+        "e2e": e2e, "gpu_launches": args.steps, "clocks": clocks, "cpu_baseline": cpu,
+        "wall_s_timed_region": round(wall, 3),
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    v.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def run_reference_draft(args, world, rank):
+    """The drafting oracle as the reference arm."""
+    if rank != 0:
+        return
+    import numpy as np
+    import torch
+    from workloads.synth import get_workload, make_inputs
+    w = get_workload(args.workload, batch=args.batch, sigma=args.sigma)
+    cores = os.cpu_count() or 1
+    per_step = max(1, min(w.batch, cores))
+    inp = make_inputs(get_workload(args.workload, batch=per_step, sigma=args.sigma),
+                      seed=args.seed, device="cpu")
+    g = torch.Generator().manual_seed(args.seed + 3000)
+    u = torch.rand(per_step, inp.parents.shape[1], generator=g)
+    with tempfile.TemporaryDirectory() as td:
+        for k, a in (("parents", inp.parents), ("drafts", inp.draft_probs), ("uniforms", u)):
+            np.save(os.path.join(td, k + ".npy"), a.numpy())
+        jobs = [(td, b) for b in range(per_step)]
+        with _oracle_pool(cores) as pool:
+            for _ in range(args.warmup):
+                pool.map(_draft_oracle_worker, jobs, chunksize=1)
+            times = []
+            for _ in range(args.steps):
+                t0 = time.perf_counter()
+                pool.map(_draft_oracle_worker, jobs, chunksize=1)
+                times.append(time.perf_counter() - t0)
+    total = sum(times)
+    value = per_step * args.steps / total
+    print(json.dumps({
+        "impl": "reference",
+        "metric": "drafted trees/sec (every node's children drawn without replacement from "
+                  "its draft row, Definition 1) and draft-row GB/s, 1 GB300",
+        "value": round(value, 4), "unit": "trees/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(total / args.steps * 1e3, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": w.name, "pipeline": "draft", "batch": w.batch, "vocab": w.vocab,
+                   "nodes": w.nodes},
+        "cpu_baseline": {"value": round(value, 4), "unit": "trees/s", "cores": cores,
+                         "kind": "oracle",
+                         "sample": f"{per_step} trees of the workload per step, one per "
+                                   f"single-threaded spawn worker"},
+        "e2e": {"value": round(value, 4), "unit": "trees/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }), flush=True)
 
 
 if __name__ == "__main__":

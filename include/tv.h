@@ -66,7 +66,10 @@ enum {
                                   0/0 was resolved as p' = 0 (p < 1) or p' = 1 (p = 1) */
   TV_STATUS_TIMEOUT = 32u,     /* a bounded device wait gave up (not expected; the tree's
                                   outputs are -1) */
-  TV_STATUS_BAD_ROW = 64u      /* a target row the traversal needed has no finite logit */
+  TV_STATUS_BAD_ROW = 64u,     /* a target row the traversal needed has no finite logit */
+  TV_STATUS_DRAFT_EXHAUSTED = 128u  /* tv_draft_children: a node had more children than
+                                       tokens of positive draft probability left (or a
+                                       row without positive finite mass) */
 };
 
 /* Flags for tv_create.  At most one path flag may be given; with none the
@@ -220,6 +223,36 @@ int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
  */
 int tv_lm_head(tv_handle* h, int M, int K, const void* hidden, const void* weight,
                float temperature, void* out_logits, float* out_row_stats, void* cuda_stream);
+
+/*
+ * tv_draft_children -- the draft side of the tree (Definition 1): every node's
+ * token drawn from its parent's draft distribution without replacement, the
+ * children of a node in index order (the order the verification tests them).
+ * Node c >= 1 with parent p takes uniforms[b][c] and gets the smallest token y
+ * (ascending token order) with u W < CDF'(y), where CDF' is the cumulative
+ * sum of draft_probs[b][p] with the tokens of p's earlier children removed and
+ * W its total.  Deterministic given the inputs, so a caller drafting level by
+ * level may call it on the tree drafted so far (rows of the new level's
+ * parents filled in) and get the same tokens for the earlier levels.
+ *   parents      [B][N+1] int32, as tv_verify_batch.
+ *   draft_probs  [B][N+1][V] fp32 (V = the handle's vocab), rows of nodes
+ *                without children are never read; 16-byte aligned rows read
+ *                four tokens a load (V % 4 == 0), any alignment works.
+ *   uniforms     [B][N+1] fp32 in [0, 1); column c draws node c, column 0 unused.
+ *   out_tokens   [B][N+1] int32: entry 0 is 0 (the root's own token is not
+ *                drawn here), entry c the token of node c, usable as
+ *                tv_verify_batch's draft_tokens.
+ * A tree with invalid parents gets -1 for every node (TV_STATUS_BAD_TREE).  A
+ * node with more children than tokens of positive mass gets -1 for the
+ * children that find none (TV_STATUS_DRAFT_EXHAUSTED).  The cumulative sums
+ * are float64 over float32 tile sums: a draw within about 1e-6 W of a step
+ * may fall on the neighbouring token.
+ * Errors: TV_ERR_INVALID_ARG, TV_ERR_CAPACITY, TV_ERR_VOCAB (a draft row too
+ * long for one CTA's shared memory, above about 600k tokens), TV_ERR_CUDA.
+ */
+int tv_draft_children(tv_handle* h, int B, int N, const int32_t* parents,
+                      const float* draft_probs, const float* uniforms, int32_t* out_tokens,
+                      void* cuda_stream);
 
 /*
  * tv_verify_batch_stats -- tv_verify_batch with the target rows' normalisers

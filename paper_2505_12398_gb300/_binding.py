@@ -20,6 +20,7 @@ TV_STATUS = {
     "DEGENERATE": 16,
     "TIMEOUT": 32,
     "BAD_ROW": 64,
+    "DRAFT_EXHAUSTED": 128,
 }
 
 
@@ -50,6 +51,7 @@ _SIGS = {
     "tv_verify_batch_stats": (_I, [_P, _I, _I, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P, _P, _P,
                                    _P]),
     "tv_lm_head": (_I, [_P, _I, _I, _P, _P, _F, _P, _P, _P]),
+    "tv_draft_children": (_I, [_P, _I, _I, _P, _P, _P, _P, _P]),
     "tv_get_status": (_I, [_P, ctypes.POINTER(ctypes.c_uint32)]),
     "tv_debug_withhold_job": (_I, [_P, _I]),
     "tv_destroy": (_I, [_P]),
@@ -210,6 +212,25 @@ class Verifier:
         if rc != 0:
             raise LibraryError("tv_lm_head", rc, self.lib)
         return logits, row_stats
+
+    def draft_children(self, parents, drafts, uniforms, out=None, stream=None):
+        """Tokens [B, N+1] int32 of every node, drawn from its parent's draft
+        row without its earlier siblings' tokens (Definition 1), node c with
+        uniforms[:, c] (tv_draft_children).  parents [B, N+1] int32, drafts
+        [B, N+1, V] fp32, uniforms [B, N+1] fp32, all on the handle's device."""
+        import torch
+        B, R = parents.shape
+        for t, dt, shape in ((parents, torch.int32, (B, R)), (drafts, torch.float32, (B, R, self.vocab)),
+                             (uniforms, torch.float32, (B, R))):
+            if t.dtype != dt or tuple(t.shape) != shape or not t.is_contiguous() \
+                    or t.device != self.device:
+                raise ValueError(f"expected a contiguous {dt} {shape} tensor on {self.device}")
+        tokens = torch.empty(B, R, dtype=torch.int32, device=self.device) if out is None else out
+        rc = self.lib.tv_draft_children(self.handle, B, R - 1, _ptr(parents), _ptr(drafts),
+                                        _ptr(uniforms), _ptr(tokens), _stream_ptr(stream))
+        if rc != 0:
+            raise LibraryError("tv_draft_children", rc, self.lib)
+        return tokens
 
     def verify_stats(self, parents, tokens, logits, drafts, temperature, uniforms, row_stats,
                      out=None, stream=None, debug=False):

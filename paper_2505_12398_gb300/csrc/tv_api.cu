@@ -399,6 +399,23 @@ int tv_lm_head(tv_handle* h, int M, int K, const void* hidden, const void* weigh
   return rc == 0 ? TV_OK : TV_ERR_CUDA;
 }
 
+int tv_draft_children(tv_handle* h, int B, int N, const int32_t* parents,
+                      const float* draft_probs, const float* uniforms, int32_t* out_tokens,
+                      void* cuda_stream) {
+  if (!h || B < 0 || N < 0) return TV_ERR_INVALID_ARG;
+  if (B > h->max_batch || N > h->max_nodes) return TV_ERR_CAPACITY;
+  if (tv_draft_smem_bytes(N, h->vocab) > 48u * 1024u) return TV_ERR_VOCAB;
+  if (B == 0) return TV_OK;
+  if (!parents || !draft_probs || !uniforms || !out_tokens ||
+      (reinterpret_cast<uintptr_t>(draft_probs) & 3u))
+    return TV_ERR_INVALID_ARG;
+  DeviceGuard guard(h->device);
+  if (!guard.ok()) return TV_ERR_CUDA;
+  const int rc = tv_launch_draft(parents, draft_probs, uniforms, out_tokens, B, N, h->vocab,
+                                 h->status, static_cast<cudaStream_t>(cuda_stream));
+  return rc == 0 ? TV_OK : TV_ERR_CUDA;
+}
+
 int tv_debug_withhold_job(tv_handle* h, int tree) {
   if (!h || tree < 0 || tree >= h->max_batch) return TV_ERR_INVALID_ARG;
   h->withhold_tree = tree;

@@ -126,3 +126,11 @@ int tv_launch_lm_head(const void* hidden, const void* weight, int M, int K, int 
                       float c_lo, void* logits, float2* part, float2* row_stats,
                       uint32_t* status, cudaStream_t stream);
 
+// Dynamic shared memory of one drafting CTA (tv_launch_draft) for N, V.
+size_t tv_draft_smem_bytes(int N, int V);
+// tokens[B][N+1]: every node's token drawn from its parent's draft row without
+// the tokens of its earlier siblings (Definition 1), uniforms[b][c] for node c;
+// one CTA per (tree, row).  0 or -5 (launch failed).
+int tv_launch_draft(const int32_t* parents, const float* drafts, const float* uniforms,
+                    int32_t* tokens, int B, int N, int V, uint32_t* status, cudaStream_t stream);
+
