@@ -9,9 +9,9 @@
 // the verification tests them.
 //
 // One CTA per (tree, row); rows without children return at once.  The CTA
-// streams its row once: each warp reduces 256-token tiles (8 tokens a lane)
-// to a float32 tile sum, and one warp turns the tile sums into a float64
-// inclusive prefix.  Each child then
+// streams its row once: each warp reduces 256-token tiles (8 tokens a lane,
+// four tiles in flight) to float32 tile sums, and one warp turns the tile
+// sums into a float64 inclusive prefix.  Each child then
 //   * finds the first tile whose prefix, less the masses of the earlier
 //     siblings' tokens up to that tile, exceeds u W (all threads, a few tiles
 //     each), and
@@ -125,12 +125,20 @@ __global__ void __launch_bounds__(kThreads)
 
   // ---- stream the row once: float32 sums of 256-token tiles
   const float* q = drafts + ((size_t)b * R + i) * (size_t)V;
-  for (int t = warp; t < n_tiles; t += kWarps) {
-    float v[8];
-    load8<kVec>(q, t * kTile + lane * 8, V, v);
-    const float s = ((v[0] + v[1]) + (v[2] + v[3])) + ((v[4] + v[5]) + (v[6] + v[7]));
-    const float ts = warp_sum_f(s);
-    if (lane == 0) tsum[t] = ts;
+  // four tiles a warp per step with 16-byte loads (loads past the end read as
+  // zeros), so that enough bytes are in flight to stream at the copy bandwidth
+  constexpr int kU = kVec ? 4 : 1;
+  for (int t = warp; t < n_tiles; t += kU * kWarps) {
+    float v[kU][8];
+#pragma unroll
+    for (int k = 0; k < kU; ++k) load8<kVec>(q, (t + k * kWarps) * kTile + lane * 8, V, v[k]);
+#pragma unroll
+    for (int k = 0; k < kU; ++k) {
+      const float s = ((v[k][0] + v[k][1]) + (v[k][2] + v[k][3])) +
+                      ((v[k][4] + v[k][5]) + (v[k][6] + v[k][7]));
+      const float ts = warp_sum_f(s);
+      if (lane == 0 && t + k * kWarps < n_tiles) tsum[t + k * kWarps] = ts;
+    }
   }
   __syncthreads();
   // float64 inclusive prefix of the tile sums (warp 0: a run of tiles a lane)
