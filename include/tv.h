@@ -152,6 +152,12 @@ int tv_create(tv_handle** out, int device, int vocab, int max_nodes, int max_bat
  *                    target distribution: its original M_b for an original
  *                    leaf, else the residual left by Eqs. (1)-(3); -1 if invalid.
  *   cuda_stream      cudaStream_t the work is queued on.
+ * CUDA graphs: the call may be captured.  A launch of the persistent kernel
+ * carries the call's queue epoch and must not be replayed, so while
+ * cuda_stream is capturing, a handle that picks its path itself verifies with
+ * the cluster path (else the three-kernel path), and a handle created with
+ * TV_FLAG_PERSISTENT returns TV_ERR_INVALID_ARG.  Make one call outside the
+ * capture first: first calls set kernel attributes and allocate scratch.
  * Errors (host-side, nothing launched): TV_ERR_INVALID_ARG, TV_ERR_TEMPERATURE,
  * TV_ERR_CAPACITY; TV_ERR_CUDA if a launch fails.  B = 0 is a no-op.
  */
@@ -261,7 +267,8 @@ int tv_draft_children(tv_handle* h, int B, int N, const int32_t* parents,
  * temperature), so no row is streamed to normalise it.  out_node_p and
  * out_stats are optional (NULL) and have the layouts of tv_verify_batch_debug
  * (out_stats[b][4], rows normalised by this call, is then 0).  Runs on the
- * persistent kernel only: other paths return TV_ERR_INVALID_ARG.
+ * persistent kernel only: other paths, and calls on a capturing stream, return
+ * TV_ERR_INVALID_ARG.
  * Errors: those of tv_verify_batch.
  */
 int tv_verify_batch_stats(tv_handle* h, int B, int N, const int32_t* parents,

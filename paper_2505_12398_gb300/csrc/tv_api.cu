@@ -94,6 +94,16 @@ class DeviceGuard {
   bool switched_ = false;
 };
 
+// True while `st` is capturing a CUDA graph.
+bool capturing(cudaStream_t st) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(st, &cs) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return cs == cudaStreamCaptureStatusActive;
+}
+
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 size_t logit_bytes(const tv_handle* h) { return h->dtype == TV_BF16 ? 2 : 4; }
@@ -151,13 +161,22 @@ int verify_impl(tv_handle* h, int B, int N, const int32_t* parents, const int32_
   if (grid > rows) grid = rows;
   if (grid < 1) grid = 1;
   FusedPlan plan;
-  const Path path = choose_path(h, B, N + 1, &plan);
+  Path path = choose_path(h, B, N + 1, &plan);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (path == kPathPersistent && capturing(st)) {
+    // a launch of the persistent kernel carries the call's queue epoch, so a
+    // graph must not replay it: under capture, a handle that chose the path
+    // itself uses the cluster path (else the three-kernel one)
+    if ((h->flags & TV_FLAG_PERSISTENT) || row_stats) return TV_ERR_INVALID_ARG;
+    plan = tv_fused_plan(B, N + 1, h->vocab, h->sm_count, h->smem_per_sm, h->smem_per_block,
+                         h->force_ncw, h->force_c, h->force_stages);
+    path = plan.ok ? kPathCluster : kPathThree;
+  }
   // the three-kernel path implements Traversal Verification only
   if (path == kPathThree && a.token_level) return TV_ERR_INVALID_ARG;
   // given row normalisers are read by the persistent kernel only
   if (row_stats && path != kPathPersistent) return TV_ERR_INVALID_ARG;
   const int bf16 = h->dtype == TV_BF16 ? 1 : 0;
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
   cudaEvent_t* ev = h->timing ? h->ev : nullptr;
   if (path == kPathCluster) {
     rc = tv_launch_fused(a, bf16, plan, st, ev);

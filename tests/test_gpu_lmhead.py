@@ -160,3 +160,55 @@ def test_lm_head_then_verification(tv):
     summ = compare_batch(det, path.cpu().numpy(), tau.cpu().numpy(), bonus.cpu().numpy(),
                          node_p.cpu().numpy(), stats.cpu().numpy())
     assert not summ["bad"], summ["bad"][:5]
+
+
+def test_token_level_with_given_normalisers(tv):
+    """The token-level verifier on the given-normaliser kernel matches its
+    oracle."""
+    from oracle.tokenlevel import verify_batch_token_level
+    w = get_workload("eagle_v32k", batch=32)
+    inp = make_inputs(w, seed=42, device="cuda")
+    B, R = inp.parents.shape
+    lf = inp.logits.double()
+    m = lf.max(dim=-1).values
+    s = torch.exp2((lf - m[..., None]) * (lmhead.LOG2E / inp.temperature)).sum(dim=-1)
+    row_stats = torch.stack([m, s], dim=-1).float().contiguous()
+    del lf
+    v = tv.Verifier(w.vocab, R - 1, B, "bf16", path="persistent", method="token")
+    path, tau, bonus, node_p, stats = v.verify_stats(
+        inp.parents, inp.tokens, inp.logits, inp.draft_probs, inp.temperature, inp.uniforms,
+        row_stats, debug=True)
+    torch.cuda.synchronize()
+    assert v.status() & ~16 == 0
+    v.close()
+    assert (stats[:, 4] == 0).all()
+    par, tok, lg, dp, un = to_numpy_inputs(inp)
+    _, _, _, det = verify_batch_token_level(par, tok, lg, dp, inp.temperature, un, keep_cdf=True)
+    summ = compare_batch(det, path.cpu().numpy(), tau.cpu().numpy(), bonus.cpu().numpy(),
+                         node_p.cpu().numpy(), stats.cpu().numpy())
+    assert not summ["bad"], summ["bad"][:5]
+
+
+def test_new_entry_points_argument_errors(tv):
+    """Host-side checks of tv_draft_children and tv_verify_batch_stats."""
+    import ctypes
+    v = tv.Verifier(1000, 7, 4, "bf16", path="three")
+    lib, h = v.lib, v.handle
+    par = torch.zeros(4, 8, dtype=torch.int32, device="cuda")
+    dr = torch.zeros(4, 8, 1000, dtype=torch.float32, device="cuda")
+    u = torch.zeros(4, 8, dtype=torch.float32, device="cuda")
+    out = torch.zeros(4, 8, dtype=torch.int32, device="cuda")
+    P = lambda t: ctypes.c_void_p(t.data_ptr())
+    assert lib.tv_draft_children(h, 5, 7, P(par), P(dr), P(u), P(out), None) == \
+        -4  # TV_ERR_CAPACITY
+    assert lib.tv_draft_children(h, 4, 8, P(par), P(dr), P(u), P(out), None) == \
+        -4  # TV_ERR_CAPACITY
+    assert lib.tv_draft_children(h, 4, 7, None, P(dr), P(u), P(out), None) == \
+        -1  # TV_ERR_INVALID_ARG
+    assert lib.tv_draft_children(h, 0, 7, None, None, None, None, None) == 0
+    # given normalisers need the persistent kernel
+    lg = torch.zeros(4, 8, 1000, dtype=torch.bfloat16, device="cuda")
+    st = torch.ones(32, 2, dtype=torch.float32, device="cuda")
+    with pytest.raises(tv.LibraryError):
+        v.verify_stats(par, out, lg, dr, 1.0, torch.zeros(4, 9, device="cuda"), st)
+    v.close()
