@@ -10,6 +10,8 @@
 #include <cstdlib>
 #include <new>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "../../include/tv.h"
 #include "tv_launch.h"
 
@@ -92,6 +94,16 @@ class DeviceGuard {
   int prev_ = 0;
   bool ok_ = false;
   bool switched_ = false;
+};
+
+// An NVTX range named after the entry point, for timeline tools (a few
+// nanoseconds when no tool is attached).
+class NvtxRange {
+ public:
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
 };
 
 // True while `st` is capturing a CUDA graph.
@@ -284,6 +296,7 @@ int tv_verify_batch(tv_handle* h, int B, int N, const int32_t* parents,
                     const float* draft_probs, float temperature, const float* uniforms,
                     int32_t* out_accepted_path, int32_t* out_accept_len,
                     int32_t* out_bonus_token, void* cuda_stream) {
+  NvtxRange range("tv_verify_batch");
   return verify_impl(h, B, N, parents, draft_tokens, target_logits, draft_probs, temperature,
                      uniforms, out_accepted_path, out_accept_len, out_bonus_token, nullptr,
                      nullptr, cuda_stream);
@@ -295,6 +308,7 @@ int tv_verify_batch_debug(tv_handle* h, int B, int N, const int32_t* parents,
                           const float* uniforms, int32_t* out_accepted_path,
                           int32_t* out_accept_len, int32_t* out_bonus_token,
                           float* out_node_p, int32_t* out_stats, void* cuda_stream) {
+  NvtxRange range("tv_verify_batch_debug");
   return verify_impl(h, B, N, parents, draft_tokens, target_logits, draft_probs, temperature,
                      uniforms, out_accepted_path, out_accept_len, out_bonus_token, out_node_p,
                      out_stats, cuda_stream);
@@ -306,6 +320,7 @@ int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
                          const float* uniforms, int32_t* out_accepted_path,
                          int32_t* out_accept_len, int32_t* out_bonus_token,
                          void* cuda_stream) {
+  NvtxRange range("tv_verify_batch_host");
   int rc = check_call(h, B, N, parents, draft_tokens, target_logits, draft_probs, temperature,
                       uniforms, out_accepted_path, out_accept_len, out_bonus_token, false);
   if (rc != TV_OK || B == 0) return rc;
@@ -378,6 +393,7 @@ int tv_verify_batch_stats(tv_handle* h, int B, int N, const int32_t* parents,
                           const float* row_stats, int32_t* out_accepted_path,
                           int32_t* out_accept_len, int32_t* out_bonus_token, float* out_node_p,
                           int32_t* out_stats, void* cuda_stream) {
+  NvtxRange range("tv_verify_batch_stats");
   if (!row_stats || (reinterpret_cast<uintptr_t>(row_stats) & 7u)) return TV_ERR_INVALID_ARG;
   return verify_impl(h, B, N, parents, draft_tokens, target_logits, draft_probs, temperature,
                      uniforms, out_accepted_path, out_accept_len, out_bonus_token, out_node_p,
@@ -386,6 +402,7 @@ int tv_verify_batch_stats(tv_handle* h, int B, int N, const int32_t* parents,
 
 int tv_lm_head(tv_handle* h, int M, int K, const void* hidden, const void* weight,
                float temperature, void* out_logits, float* out_row_stats, void* cuda_stream) {
+  NvtxRange range("tv_lm_head");
   if (!h || M < 0 || K < 64 || (K % 64) != 0) return TV_ERR_INVALID_ARG;
   if (h->dtype != TV_BF16 || (h->vocab % 8) != 0) return TV_ERR_INVALID_ARG;
   if ((size_t)M > (size_t)h->max_batch * (h->max_nodes + 1)) return TV_ERR_CAPACITY;
@@ -421,6 +438,7 @@ int tv_lm_head(tv_handle* h, int M, int K, const void* hidden, const void* weigh
 int tv_draft_children(tv_handle* h, int B, int N, const int32_t* parents,
                       const float* draft_probs, const float* uniforms, int32_t* out_tokens,
                       void* cuda_stream) {
+  NvtxRange range("tv_draft_children");
   if (!h || B < 0 || N < 0) return TV_ERR_INVALID_ARG;
   if (B > h->max_batch || N > h->max_nodes) return TV_ERR_CAPACITY;
   if (tv_draft_smem_bytes(N, h->vocab) > 48u * 1024u) return TV_ERR_VOCAB;
