@@ -44,11 +44,13 @@ def parse_args():
                          "(top-down RRS without replacement) verifier it is compared with")
     ap.add_argument("--path", choices=["auto", "persistent", "cluster", "three"], default="auto",
                     help="kernel path of the handle (auto: the library's choice)")
-    ap.add_argument("--pipeline", choices=["verify", "lmhead", "draft"], default="verify",
+    ap.add_argument("--pipeline", choices=["verify", "lmhead", "draft", "full"],
+                    default="verify",
                     help="verify: one step = one verification call; lmhead: one step = the "
                          "target LM head (logits and row normalisers on the tensor cores) "
                          "followed by verification with those normalisers; draft: one step = "
-                         "drafting every node's children without replacement")
+                         "drafting every node's children without replacement; full: drafting, "
+                         "then the LM head, then verification")
     ap.add_argument("--hidden", type=int, default=4096,
                     help="hidden size K of the LM head (--pipeline lmhead)")
     ap.add_argument("--e2e-steps", type=int, default=10)
@@ -276,12 +278,12 @@ def main():
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
 
     if args.impl == "reference":
-        if args.pipeline == "lmhead":
+        if args.pipeline in ("lmhead", "full"):
             return run_reference_lmhead(args, world, rank)
         if args.pipeline == "draft":
             return run_reference_draft(args, world, rank)
         return run_reference(args, world, rank)
-    if args.pipeline == "lmhead":
+    if args.pipeline in ("lmhead", "full"):
         return main_lmhead(args, world, rank, local_rank)
     if args.pipeline == "draft":
         return main_draft(args, world, rank, local_rank)
@@ -532,7 +534,7 @@ def run_reference(args, world, rank):
 
 # ------------------------------------------------- LM-head pipeline ---------
 
-def dump_lmhead_sample(lin, trees, tmpdir):
+def dump_lmhead_sample(lin, trees, tmpdir, u_draft=None):
     """Host copies, for the oracle, of the sampled trees' hidden states and
     draft side, and of the output embedding (bf16 bit patterns)."""
     import numpy as np
@@ -549,6 +551,8 @@ def dump_lmhead_sample(lin, trees, tmpdir):
         "parents": inp.parents[idx].cpu().numpy(), "tokens": inp.tokens[idx].cpu().numpy(),
         "drafts": inp.draft_probs[idx].cpu().numpy(), "uniforms": inp.uniforms[idx].cpu().numpy(),
     }
+    if u_draft is not None:
+        arrays["udraft"] = u_draft[idx].cpu().numpy()
     for k, a in arrays.items():
         np.save(os.path.join(outdir, k + ".npy"), a)
     return outdir
@@ -577,7 +581,12 @@ def _lmhead_oracle_worker(args):
         v1 = min(V, v0 + step)
         logits[:, v0:v1] = lmhead.logits(h, _bf16_bits_to_f64(np.asarray(wt[v0:v1])))
     stored = lmhead.to_bf16(logits)
-    r = verify_tree(d["parents"][b], d["tokens"][b], stored, d["drafts"][b], temperature,
+    tokens = d["tokens"][b]
+    if "udraft" in d.d:                # the full pipeline drafts the tree first
+        from oracle.drafting import sample_tree
+        tokens = np.asarray(sample_tree(d["parents"][b], d["drafts"][b],
+                                        [float(x) for x in d["udraft"][b]]))
+    r = verify_tree(d["parents"][b], tokens, stored, d["drafts"][b], temperature,
                     d["uniforms"][b])
     return r["tau"]
 
@@ -597,9 +606,18 @@ def _oracle_pool(cores):
     return mp.get_context("spawn").Pool(cores)
 
 
+LMHEAD_METRIC = {
+    "lmhead": "verified trees/sec including the target LM head (logits + row normalisers on "
+              "the tensor cores, then verification), 1 GB300",
+    "full": "drafted and verified trees/sec (drafting without replacement, the target LM "
+            "head with its row normalisers, then verification), 1 GB300",
+}
+
+
 def main_lmhead(args, world, rank, local_rank):
     """One step = tv_lm_head (logits and row normalisers of every row of the
-    batch, tensor cores) then tv_verify_batch_stats on them."""
+    batch, tensor cores) then tv_verify_batch_stats on them; with --pipeline
+    full, tv_draft_children first draws the trees' tokens."""
     import torch
     import torch.distributed as dist
     import paper_2505_12398_gb300 as tv
@@ -628,17 +646,30 @@ def main_lmhead(args, world, rank, local_rank):
     out = (torch.empty(B, N, dtype=torch.int32, device=dev),
            torch.empty(B, dtype=torch.int32, device=dev),
            torch.empty(B, dtype=torch.int32, device=dev))
+    full = args.pipeline == "full"
+    gd = torch.Generator(device=dev).manual_seed(rank_seed(args.seed, rank) + 3000)
+    u_draft = torch.rand(B, R, generator=gd, device=dev)
+    tokens = torch.empty(B, R, dtype=torch.int32, device=dev)
+    # the per-step input besides hidden states and the draft side: the drafting
+    # uniforms (full pipeline) or the draft tokens
+    side0 = u_draft if full else inp.tokens
 
-    def step():
-        v.lm_head(lin.hidden, lin.weight, inp.temperature, out=lm_out, stream=stream)
-        v.verify_stats(inp.parents, inp.tokens, logits, inp.draft_probs, inp.temperature,
-                       inp.uniforms, row_stats, out=out, stream=stream)
+    def step(ev=None, hidden=lin.hidden, parents=inp.parents, drafts=inp.draft_probs,
+             uniforms=inp.uniforms, side=side0, debug=False):
+        toks = side
+        if full:
+            v.draft_children(parents, drafts, side, out=tokens, stream=stream)
+            toks = tokens
+        if ev is not None:
+            ev[1].record(stream)
+        v.lm_head(hidden, lin.weight, inp.temperature, out=lm_out, stream=stream)
+        if ev is not None:
+            ev[2].record(stream)
+        return v.verify_stats(parents, toks, logits, drafts, inp.temperature, uniforms,
+                              row_stats, out=None if debug else out, stream=stream, debug=debug)
 
     # instrumented call: the rows each tree reads, tau
-    v.lm_head(lin.hidden, lin.weight, inp.temperature, out=lm_out, stream=stream)
-    _, tau_d, _, _, stats = v.verify_stats(inp.parents, inp.tokens, logits, inp.draft_probs,
-                                           inp.temperature, inp.uniforms, row_stats,
-                                           stream=stream, debug=True)
+    _, tau_d, _, _, stats = step(debug=True)
     torch.cuda.synchronize(dev)
     if v.status() & ~16:
         raise RuntimeError(f"device status {tv.status_names(v.status())}")
@@ -661,31 +692,29 @@ def main_lmhead(args, world, rank, local_rank):
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize(dev)
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
     wall0 = time.perf_counter()
     for k in range(args.steps):
         flush.zero_()
         ev[k][0].record(stream)
-        v.lm_head(lin.hidden, lin.weight, inp.temperature, out=lm_out, stream=stream)
-        ev[k][1].record(stream)
-        v.verify_stats(inp.parents, inp.tokens, logits, inp.draft_probs, inp.temperature,
-                       inp.uniforms, row_stats, out=out, stream=stream)
-        ev[k][2].record(stream)
+        step(ev[k])
+        ev[k][3].record(stream)
     torch.cuda.synchronize(dev)
     wall = time.perf_counter() - wall0
     if world > 1:
         dist.barrier()
     clocks = sampler.stop()
-    gemm_ms = sum(e[0].elapsed_time(e[1]) for e in ev) / args.steps
-    ver_ms = sum(e[1].elapsed_time(e[2]) for e in ev) / args.steps
-    total_ms = sum(e[0].elapsed_time(e[2]) for e in ev)
+    draft_ms = sum(e[0].elapsed_time(e[1]) for e in ev) / args.steps
+    gemm_ms = sum(e[1].elapsed_time(e[2]) for e in ev) / args.steps
+    ver_ms = sum(e[2].elapsed_time(e[3]) for e in ev) / args.steps
+    total_ms = sum(e[0].elapsed_time(e[3]) for e in ev)
     total_ms_max = max_over_ranks(total_ms, world, dev)
 
     # end to end: hidden states and the draft side from pinned host memory,
     # outputs back to the host, every step
     e2e = None
     if not args.no_e2e:
-        hp = [x.cpu().pin_memory() for x in (lin.hidden, inp.parents, inp.tokens,
+        hp = [x.cpu().pin_memory() for x in (lin.hidden, inp.parents, side0,
                                               inp.draft_probs, inp.uniforms)]
         dbuf = [torch.empty_like(x, device=dev) for x in hp]
         hout = [torch.empty(o.shape, dtype=o.dtype).pin_memory() for o in out]
@@ -693,9 +722,8 @@ def main_lmhead(args, world, rank, local_rank):
         def e2e_step():
             for d, h in zip(dbuf, hp):
                 d.copy_(h, non_blocking=True)
-            v.lm_head(dbuf[0], lin.weight, inp.temperature, out=lm_out, stream=stream)
-            v.verify_stats(dbuf[1], dbuf[2], logits, dbuf[3], inp.temperature, dbuf[4],
-                           row_stats, out=out, stream=stream)
+            step(hidden=dbuf[0], parents=dbuf[1], side=dbuf[2], drafts=dbuf[3],
+                 uniforms=dbuf[4])
             for h, o in zip(hout, out):
                 h.copy_(o, non_blocking=True)
 
@@ -720,7 +748,7 @@ def main_lmhead(args, world, rank, local_rank):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline_lmhead(lin, args, B)
+        cpu = cpu_baseline_lmhead(lin, args, B, u_draft if full else None)
 
     peak, peak_kind = measured_bf16_peak()
     hbm, hbm_kind = measured_peaks()
@@ -728,22 +756,24 @@ def main_lmhead(args, world, rank, local_rank):
     gemm_tflops = flops / (gemm_ms / 1e3) / 1e12
     ver_gbs = trav_bytes / (ver_ms / 1e3) / 1e9
     ms_step = total_ms_max / args.steps
+    phases = {"lm_head_kernel+lm_head_merge_kernel": round(gemm_ms, 6),
+              "tv_flow_kernel (given normalisers)": round(ver_ms, 6)}
+    if full:
+        phases = {"tv_draft_kernel": round(draft_ms, 6), **phases}
     line = {
-        "metric": "verified trees/sec including the target LM head (logits + row "
-                  "normalisers on the tensor cores, then verification), 1 GB300",
+        "metric": LMHEAD_METRIC[args.pipeline],
         "value": round(whole_job_rate(B, world, args.steps, total_ms_max), 3),
         "unit": "trees/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(ms_step, 6), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (hidden states and output embedding whose product has the "
                 "workload's logit law; draft side drawn from those logits)",
-        "config": {"workload": w.name, "pipeline": "lmhead", "batch": B, "vocab": V,
+        "config": {"workload": w.name, "pipeline": args.pipeline, "batch": B, "vocab": V,
                    "nodes": N, "hidden": K, "rows": M, "method": args.method,
                    "temperature": w.temperature, "sigma": w.sigma, "seed": args.seed,
                    "l2": "flushed by a 256 MiB write before every timed step (untimed)",
                    "parallelism": f"dp{world} (independent trees per GPU)"},
-        "phase_ms": {"lm_head_kernel+lm_head_merge_kernel": round(gemm_ms, 6),
-                     "tv_flow_kernel (given normalisers)": round(ver_ms, 6)},
+        "phase_ms": phases,
         "mean_accept_len_tau_plus_1": round(mean_tau1, 4),
         "roofline": {"bound": "tensor", "kernel": "lm_head_kernel",
                      "achieved": round(gemm_tflops, 2), "peak": peak, "unit": "TFLOP/s",
@@ -755,7 +785,7 @@ def main_lmhead(args, world, rank, local_rank):
                             "frac": round(ver_gbs / hbm, 4), "peak_kind": hbm_kind,
                             "bytes_per_launch": trav_bytes},
         "e2e": e2e,
-        "gpu_launches": 3 * args.steps,
+        "gpu_launches": (4 if full else 3) * args.steps,
         "clocks": clocks,
         "cpu_baseline": cpu,
         "wall_s_timed_region": round(wall, 3),
@@ -767,18 +797,19 @@ def main_lmhead(args, world, rank, local_rank):
         dist.destroy_process_group()
 
 
-def cpu_baseline_lmhead(lin, args, B):
+def cpu_baseline_lmhead(lin, args, B, u_draft=None):
     cores = os.cpu_count() or 1
     with tempfile.TemporaryDirectory() as td:
         n_sample = min(B, cores)
-        sdir = dump_lmhead_sample(lin, range(n_sample), td)
+        sdir = dump_lmhead_sample(lin, range(n_sample), td, u_draft)
         with _oracle_pool(cores) as pool:
             t_probe, _, _ = time_lmhead_oracle(sdir, n_sample, lin.inputs.temperature, pool)
             reps = max(1, min(50, int(args.cpu_seconds / max(t_probe, 1e-3))))
             t, n, _ = time_lmhead_oracle(sdir, n_sample, lin.inputs.temperature, pool, reps=reps)
     return {"value": round(n / t, 4), "unit": "trees/s", "cores": cores, "kind": "oracle",
             "sample": f"{n} trees ({n_sample} distinct trees of the batch, repeated {reps}x) "
-                      f"through the oracle LM head (float64 products, bf16 storage) and "
+                      + ("drafted by the oracle, " if u_draft is not None else "")
+                      + f"through the oracle LM head (float64 products, bf16 storage) and "
                       f"verification, one tree per single-threaded spawn worker, {t:.1f} s"}
 
 
@@ -794,8 +825,12 @@ def run_reference_lmhead(args, world, rank):
     gen_w = get_workload(args.workload, batch=per_step, sigma=args.sigma,
                          logit_dtype=torch.bfloat16)
     lin = make_lmhead_inputs(gen_w, hidden=args.hidden, seed=args.seed, device="cpu")
+    u_draft = None
+    if args.pipeline == "full":
+        g = torch.Generator().manual_seed(args.seed + 3000)
+        u_draft = torch.rand(per_step, lin.inputs.parents.shape[1], generator=g)
     with tempfile.TemporaryDirectory() as td:
-        sdir = dump_lmhead_sample(lin, range(per_step), td)
+        sdir = dump_lmhead_sample(lin, range(per_step), td, u_draft)
         with _oracle_pool(cores) as pool:
             for _ in range(args.warmup):
                 time_lmhead_oracle(sdir, per_step, lin.inputs.temperature, pool)
@@ -805,13 +840,12 @@ def run_reference_lmhead(args, world, rank):
     value = per_step * args.steps / total
     line = {
         "impl": "reference",
-        "metric": "verified trees/sec including the target LM head (logits + row "
-                  "normalisers on the tensor cores, then verification), 1 GB300",
+        "metric": LMHEAD_METRIC[args.pipeline],
         "value": round(value, 4), "unit": "trees/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(total / args.steps * 1e3, 3),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
-        "config": {"workload": w.name, "pipeline": "lmhead", "batch": w.batch,
+        "config": {"workload": w.name, "pipeline": args.pipeline, "batch": w.batch,
                    "vocab": w.vocab, "nodes": w.nodes, "hidden": args.hidden,
                    "method": args.method},
         "cpu_baseline": {"value": round(value, 4), "unit": "trees/s", "cores": cores,

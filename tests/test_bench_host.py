@@ -75,3 +75,31 @@ def test_lmhead_oracle_leg_matches_the_oracle_on_the_generated_logits(tmp_path):
                         inp.logits[b].float().numpy().astype(np.float64),
                         inp.draft_probs[b].numpy(), inp.temperature, inp.uniforms[b].numpy())
         assert taus[b] == r["tau"]
+
+
+def test_full_pipeline_oracle_leg_drafts_first(tmp_path):
+    """With drafting uniforms in the sample, the CPU leg drafts each tree with
+    the drafting oracle before verifying it."""
+    import numpy as np
+    from oracle.drafting import sample_tree
+    from oracle.verify import verify_tree
+    from workloads.synth import get_workload, make_lmhead_inputs
+    w = get_workload("binary4", batch=3, vocab=512, logit_dtype=torch.bfloat16)
+    lin = make_lmhead_inputs(w, hidden=64, seed=5)
+    g = torch.Generator().manual_seed(10)
+    lin.hidden.copy_((torch.randint(-8, 9, lin.hidden.shape, generator=g) / 16.0).to(torch.bfloat16))
+    lin.weight.copy_((torch.randint(-8, 9, lin.weight.shape, generator=g) / 16.0).to(torch.bfloat16))
+    inp = lin.inputs
+    B, R = inp.parents.shape
+    inp.logits.copy_((lin.hidden.float() @ lin.weight.float().T).view(B, R, -1).to(torch.bfloat16))
+    u_draft = torch.rand(B, R, generator=g)
+    d = bench.dump_lmhead_sample(lin, range(B), str(tmp_path), u_draft)
+    with bench._oracle_pool(2) as pool:
+        _, n, taus = bench.time_lmhead_oracle(d, B, inp.temperature, pool)
+    for b in range(B):
+        drafts = inp.draft_probs[b].numpy()
+        toks = sample_tree(inp.parents[b].numpy(), drafts, u_draft[b].tolist())
+        r = verify_tree(inp.parents[b].numpy(), np.asarray(toks),
+                        inp.logits[b].float().numpy().astype(np.float64), drafts,
+                        inp.temperature, inp.uniforms[b].numpy())
+        assert taus[b] == r["tau"]
