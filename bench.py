@@ -386,8 +386,8 @@ def main():
         torch.cuda.synchronize(dev)
         e_ms = x0.elapsed_time(x1)
         e_ms_max = max_over_ranks(e_ms, world, dev)
-        h2d = sum(x.numel() * x.element_size() for x in hp)
-        d2h = sum(x.numel() * x.element_size() for x in hout)
+        # what the host entry point copied (it skips the draft rows of leaves)
+        h2d, d2h = v.last_host_copy_bytes()
         assert torch.equal(hout[1], out[1].cpu()), "host entry point disagrees"
         e2e = {"value": round(whole_job_rate(B, world, ks, e_ms_max), 3), "unit": "trees/s",
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": ks}

@@ -197,7 +197,9 @@ int tv_verify_batch_debug(tv_handle* h, int B, int N, const int32_t* parents,
  * by tv_create's limits), runs tv_verify_batch on cuda_stream, copies the
  * three outputs back and synchronises the stream before returning.  All
  * pointers are host pointers with the layouts above; pinned (page-locked)
- * memory gives the fastest copies.  Errors as tv_verify_batch.
+ * memory gives the fastest copies.  Draft rows of nodes without children are
+ * never read and are not copied (one 2-D copy per run of rows with children
+ * when all trees share their parents).  Errors as tv_verify_batch.
  */
 int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
                          const int32_t* draft_tokens, const void* target_logits,
@@ -205,6 +207,13 @@ int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
                          const float* uniforms, int32_t* out_accepted_path,
                          int32_t* out_accept_len, int32_t* out_bonus_token,
                          void* cuda_stream);
+
+/*
+ * tv_last_host_copy_bytes -- bytes the last successful tv_verify_batch_host
+ * call on this handle copied host to device (*h2d) and device to host (*d2h).
+ * Either pointer may be NULL.  Errors: TV_ERR_INVALID_ARG (no handle).
+ */
+int tv_last_host_copy_bytes(tv_handle* h, uint64_t* h2d, uint64_t* d2h);
 
 /*
  * tv_lm_head -- the target model's last layer fused with the row normalisers

@@ -52,6 +52,7 @@ _SIGS = {
                                    _P]),
     "tv_lm_head": (_I, [_P, _I, _I, _P, _P, _F, _P, _P, _P]),
     "tv_draft_children": (_I, [_P, _I, _I, _P, _P, _P, _P, _P]),
+    "tv_last_host_copy_bytes": (_I, [_P, _P, _P]),
     "tv_get_status": (_I, [_P, ctypes.POINTER(ctypes.c_uint32)]),
     "tv_debug_withhold_job": (_I, [_P, _I]),
     "tv_destroy": (_I, [_P]),
@@ -273,6 +274,15 @@ class Verifier:
         if rc != 0:
             raise LibraryError("tv_verify_batch_host", rc, self.lib)
         return path, tau, bonus
+
+    def last_host_copy_bytes(self):
+        """(host-to-device, device-to-host) bytes of the last verify_host call
+        (tv_last_host_copy_bytes)."""
+        h2d, d2h = ctypes.c_uint64(), ctypes.c_uint64()
+        rc = self.lib.tv_last_host_copy_bytes(self.handle, ctypes.byref(h2d), ctypes.byref(d2h))
+        if rc != 0:
+            raise LibraryError("tv_last_host_copy_bytes", rc, self.lib)
+        return h2d.value, d2h.value
 
     def set_phase_timing(self, enable=True):
         rc = self.lib.tv_set_phase_timing(self.handle, 1 if enable else 0)

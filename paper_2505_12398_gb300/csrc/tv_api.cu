@@ -8,7 +8,10 @@
 #include <cstdint>
 #include <cstdio>
 #include <cstdlib>
+#include <algorithm>
+#include <cstring>
 #include <new>
+#include <vector>
 
 #include <nvtx3/nvToolsExt.h>
 
@@ -39,9 +42,11 @@ struct tv_handle {
   // per-(row, tile) scratch of tv_lm_head (allocated on first use)
   float2* lmh_part = nullptr;
   size_t lmh_part_bytes = 0;
-  // staging for tv_verify_batch_host (allocated on first use)
+  // staging for tv_verify_batch_host (allocated on first use), and the bytes
+  // its last call copied each way
   char* stage = nullptr;
   size_t stage_bytes = 0;
+  uint64_t host_h2d_bytes = 0, host_d2h_bytes = 0;
   // optional per-kernel timing events
   bool timing = false;
   bool timed_call = false;
@@ -105,6 +110,64 @@ class NvtxRange {
   NvtxRange(const NvtxRange&) = delete;
   NvtxRange& operator=(const NvtxRange&) = delete;
 };
+
+// Copies the draft rows of nodes with children from host to device (rows of
+// leaves are never read).  When every tree has the same parents, each run of
+// consecutive rows with children is one 2-D copy over the batch; otherwise one
+// copy per run per tree.  Adds the bytes copied to *bytes.
+bool copy_draft_rows(float* dst, const float* src, const int32_t* parents, int B, size_t R,
+                     size_t V, cudaStream_t st, size_t* bytes) {
+  const size_t row = V * sizeof(float);
+  auto rows_with_children = [&](int b, std::vector<char>& kid) {
+    std::fill(kid.begin(), kid.end(), 0);
+    for (size_t i = 1; i < R; ++i) {
+      const int p = parents[(size_t)b * R + i];
+      if (p >= 0 && (size_t)p < i) kid[p] = 1;
+    }
+  };
+  auto runs = [&](const std::vector<char>& kid, auto&& copy) {
+    for (size_t r0 = 0; r0 < R;) {
+      if (!kid[r0]) {
+        ++r0;
+        continue;
+      }
+      size_t r1 = r0;
+      while (r1 < R && kid[r1]) ++r1;
+      if (!copy(r0, r1)) return false;
+      r0 = r1;
+    }
+    return true;
+  };
+  std::vector<char> kid(R);
+  bool same = true;
+  for (int b = 1; b < B && same; ++b)
+    same = std::memcmp(parents, parents + (size_t)b * R, R * sizeof(int32_t)) == 0;
+  if (same) {
+    rows_with_children(0, kid);
+    const bool ok = runs(kid, [&](size_t r0, size_t r1) {
+      if (cudaMemcpy2DAsync(dst + r0 * V, R * row, src + r0 * V, R * row, (r1 - r0) * row,
+                            (size_t)B, cudaMemcpyHostToDevice, st) != cudaSuccess)
+        return false;
+      *bytes += (r1 - r0) * row * (size_t)B;
+      return true;
+    });
+    if (ok) return true;
+    cudaGetLastError();   // (a pitch beyond the 2-D limit: copy tree by tree)
+  }
+  for (int b = 0; b < B; ++b) {
+    rows_with_children(b, kid);
+    const size_t base = (size_t)b * R;
+    if (!runs(kid, [&](size_t r0, size_t r1) {
+          if (cudaMemcpyAsync(dst + (base + r0) * V, src + (base + r0) * V, (r1 - r0) * row,
+                              cudaMemcpyHostToDevice, st) != cudaSuccess)
+            return false;
+          *bytes += (r1 - r0) * row;
+          return true;
+        }))
+      return false;
+  }
+  return true;
+}
 
 // True while `st` is capturing a CUDA graph.
 bool capturing(cudaStream_t st) {
@@ -366,8 +429,9 @@ int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
   bool ok = cudaMemcpyAsync(d_par, parents, n_tree, cudaMemcpyHostToDevice, st) == cudaSuccess &&
             cudaMemcpyAsync(d_tok, draft_tokens, n_tree, cudaMemcpyHostToDevice, st) == cudaSuccess &&
             cudaMemcpyAsync(d_unif, uniforms, n_unif, cudaMemcpyHostToDevice, st) == cudaSuccess &&
-            cudaMemcpyAsync(d_logit, target_logits, n_logit, cudaMemcpyHostToDevice, st) == cudaSuccess &&
-            cudaMemcpyAsync(d_draft, draft_probs, n_draft, cudaMemcpyHostToDevice, st) == cudaSuccess;
+            cudaMemcpyAsync(d_logit, target_logits, n_logit, cudaMemcpyHostToDevice, st) == cudaSuccess;
+  size_t draft_bytes = 0;
+  ok = ok && copy_draft_rows(d_draft, draft_probs, parents, B, R, V, st, &draft_bytes);
   if (!ok) {
     cudaGetLastError();
     return TV_ERR_CUDA;
@@ -384,6 +448,15 @@ int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
     cudaGetLastError();
     return TV_ERR_CUDA;
   }
+  h->host_h2d_bytes = 2 * n_tree + n_unif + n_logit + draft_bytes;
+  h->host_d2h_bytes = (N > 0 ? n_path : 0) + 2 * n_out;
+  return TV_OK;
+}
+
+int tv_last_host_copy_bytes(tv_handle* h, uint64_t* h2d, uint64_t* d2h) {
+  if (!h) return TV_ERR_INVALID_ARG;
+  if (h2d) *h2d = h->host_h2d_bytes;
+  if (d2h) *d2h = h->host_d2h_bytes;
   return TV_OK;
 }
 

@@ -186,6 +186,42 @@ def test_host_entry_point_matches_device(tv):
     assert (out[2].numpy() == bonus).all()
 
 
+@pytest.mark.parametrize("shapes", ["same", "random"])
+def test_host_entry_point_copies_only_needed_draft_rows(tv, shapes):
+    """The host entry point copies the draft rows of nodes with children only
+    (2-D copies when all trees share a shape, per tree otherwise).  Two calls
+    on one handle with different inputs: stale staging from the first would
+    change the second's results if a needed row were missed."""
+    from workloads.synth import make_inputs_random_shapes
+    if shapes == "same":
+        mk = lambda seed: make_inputs(get_workload("eagle_v32k", batch=24), seed=seed,
+                                      device="cuda")
+    else:
+        mk = lambda seed: make_inputs_random_shapes(24, 60, 32000, seed=seed, device="cuda")
+    first, second = mk(51), mk(52)
+    B, R = second.parents.shape
+    v = tv.Verifier(32000, R - 1, B, "bf16")
+    out = (torch.empty(B, R - 1, dtype=torch.int32), torch.empty(B, dtype=torch.int32),
+           torch.empty(B, dtype=torch.int32))
+    for inp in (first, second):
+        hp = [x.cpu() for x in (inp.parents, inp.tokens, inp.logits, inp.draft_probs,
+                                inp.uniforms)]
+        v.verify_host(hp[0], hp[1], hp[2], hp[3], inp.temperature, hp[4], out)
+    h2d, d2h = v.last_host_copy_bytes()
+    want = v.verify(second.parents, second.tokens, second.logits, second.draft_probs,
+                    second.temperature, second.uniforms)
+    torch.cuda.synchronize()
+    assert v.status() & ~16 == 0
+    v.close()
+    for a, b in zip(out, want):
+        assert torch.equal(a, b.cpu())
+    par = second.parents.cpu().numpy()
+    internal = sum(len({int(p) for p in par[b, 1:]}) for b in range(B))
+    V = 32000
+    assert h2d == 2 * B * R * 4 + B * (R + 1) * 4 + B * R * V * 2 + internal * V * 4
+    assert d2h == B * (R - 1) * 4 + 2 * B * 4
+
+
 def test_host_argument_errors(tv):
     w = get_workload("tiny", batch=2)
     inp = make_inputs(w, seed=0, device="cuda")
