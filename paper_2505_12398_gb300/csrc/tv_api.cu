@@ -61,14 +61,14 @@ constexpr unsigned kPathFlags = TV_FLAG_UNFUSED | TV_FLAG_CLUSTER | TV_FLAG_PERS
 
 enum Path { kPathThree = 0, kPathCluster = 1, kPathPersistent = 2 };
 
-FlowPlan flow_plan(const tv_handle* h, int R) {
-  return tv_flow_plan(R, h->smem_per_sm, h->smem_per_block, h->flow_force[0], h->flow_force[1],
+FlowPlan flow_plan(const tv_handle* h, int R, int B) {
+  return tv_flow_plan(R, B, h->smem_per_sm, h->smem_per_block, h->flow_force[0], h->flow_force[1],
                       h->flow_force[2], h->flow_force[3], h->flow_force[4]);
 }
 
 // Smallest slice the persistent kernel may use on this handle (sizes its queue).
 int flow_min_slice(const tv_handle* h) {
-  const FlowPlan p = flow_plan(h, h->max_nodes + 1);
+  const FlowPlan p = flow_plan(h, h->max_nodes + 1, h->max_batch);
   return p.slice_min;
 }
 
@@ -79,7 +79,7 @@ Path choose_path(const tv_handle* h, int B, int R, FusedPlan* plan) {
                           h->force_ncw, h->force_c, h->force_stages);
     return plan->ok ? kPathCluster : kPathThree;
   }
-  if (!h->flow_ws || !flow_plan(h, R).ok) return kPathThree;
+  if (!h->flow_ws || !flow_plan(h, R, B).ok) return kPathThree;
   return kPathPersistent;
 }
 
@@ -257,7 +257,7 @@ int verify_impl(tv_handle* h, int B, int N, const int32_t* parents, const int32_
     rc = tv_launch_fused(a, bf16, plan, st, ev);
   } else if (path == kPathPersistent) {
     FlowArgs f;
-    const FlowPlan fp = flow_plan(h, N + 1);
+    const FlowPlan fp = flow_plan(h, N + 1, B);
     if (tv_flow_bind(h->flow_ws, h->flow_ws_bytes, B, N + 1, h->vocab, fp, &f) != 0)
       return TV_ERR_CAPACITY;
     f.epoch = ++h->epoch;
@@ -334,7 +334,9 @@ int tv_create(tv_handle** out, int device, int vocab, int max_nodes, int max_bat
     // the queue's publication tags start at zero; calls use epochs 1, 2, ...
     // the queue is sized for the smallest slice; for very large handles the
     // smallest slice grows until the workspace stays within 1 GiB
-    const FlowPlan fp = flow_plan(h, max_nodes + 1);
+    // (bounded by the pass slice of the smallest batches, so that every call's
+    // slices stay at or above the size the queue was built for)
+    const FlowPlan fp = flow_plan(h, max_nodes + 1, 1);
     int min_slice = fp.slice_min;
     while (tv_flow_workspace_bytes(max_batch, max_nodes + 1, vocab, min_slice) > (1ull << 30) &&
            min_slice < fp.slice_pass)
@@ -586,7 +588,7 @@ int tv_launch_shape(tv_handle* h, int B, int N, int* path, int* cluster, int* wa
   const Path p = choose_path(h, B, N + 1, &plan);
   if (path) *path = (int)p;
   if (cluster) *cluster = (p == kPathCluster) ? plan.C : 1;
-  const FlowPlan fp = flow_plan(h, N + 1);
+  const FlowPlan fp = flow_plan(h, N + 1, B);
   if (warps) *warps = (p == kPathCluster) ? plan.ncw : (p == kPathPersistent ? fp.ncw : 16);
   if (stages)
     *stages = (p == kPathCluster) ? plan.stages : (p == kPathPersistent ? fp.stages : 0);

@@ -91,15 +91,15 @@ struct FlowArgs {
 struct FlowPlan {
   int ncw = 4;                   // consumer warps per CTA (4 or 8)
   int stages = 3;                // ring stages of 3 KB per consumer warp
-  int slice_pass = 8192;         // largest slice of a pass / bonus draw (tokens)
-  int slice_stats = 16384;       // largest slice of a row normaliser (tokens)
+  int slice_pass = 8192;         // largest slice of a pass / bonus draw (tokens; by batch)
+  int slice_stats = 16384;       // largest slice of a row normaliser (tokens; by batch)
   int slice_min = 2048;          // slices shrink to this as fewer trees remain
   size_t smem = 0;
   bool ok = false;
 };
 
-// Default plan for R = N+1 rows (tuning overrides: force_* > 0).
-FlowPlan tv_flow_plan(int R, int smem_per_sm, int smem_per_block, int force_ncw,
+// Default plan for R = N+1 rows and B trees (tuning overrides: force_* > 0).
+FlowPlan tv_flow_plan(int R, int B, int smem_per_sm, int smem_per_block, int force_ncw,
                       int force_stages, int force_slice_pass, int force_slice_stats,
                       int force_slice_min);
 // Workspace for slices of at least `min_slice` tokens.

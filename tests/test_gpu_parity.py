@@ -116,6 +116,14 @@ def test_default_launch_shapes(tv, batch, path):
     check(tv, inp, trees=trees, path=path)
 
 
+def test_eagle_v128k_large_batch_sampled(tv):
+    """1024 trees of 128256 tokens: the persistent kernel's largest slices
+    (32768 tokens, several per row), sampled trees against the oracle."""
+    w = get_workload("eagle_v128k", batch=1024)
+    inp = make_inputs(w, seed=9, device="cuda")
+    check(tv, inp, trees=list(range(0, 1024, 64)), path="persistent")
+
+
 @pytest.mark.parametrize("V", [1000, 1003, 257, 8, 8200, 16392])
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
 @pytest.mark.parametrize("path", ["auto", "cluster"])
