@@ -10,6 +10,11 @@ timed interval.  Times are CUDA-event device times on the launching stream.
 Prints ONE JSON line (rank 0).  ``--impl reference`` times the CPU oracle
 (the slow literal float64 restatement of the paper's algorithm) on the host
 cores instead, on a bounded sample of the same workload per step.
+
+``--pipeline`` times the steps on either side of the verification as well:
+``draft`` (drawing every node's children without replacement, Definition 1),
+``lmhead`` (the target's logits and row normalisers on the tensor cores, then
+verification with them) and ``full`` (drafting, LM head, verification).
 """
 
 import argparse
