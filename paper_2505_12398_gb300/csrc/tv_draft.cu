@@ -69,7 +69,7 @@ __device__ __forceinline__ void load8(const float* __restrict__ q, int x0, int V
   }
 }
 
-// Tree blockIdx.x, row blockIdx.y.  Dynamic shared memory (tv_draft_smem_bytes):
+// Tree blockIdx.x, row blockIdx.y.  Dynamic shared memory (draft_smem_bytes):
 // pre[n_tiles] f64, rem_q[R] f64, tsum[n_tiles] f32, par[R], kids[R],
 // rem_tok[R] int32.
 template <bool kVec>
