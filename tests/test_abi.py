@@ -54,3 +54,40 @@ def test_product_path_does_not_import_the_oracle():
             if f.endswith((".py", ".cu", ".cuh", ".h")):
                 text = open(os.path.join(dirpath, f)).read()
                 assert "import oracle" not in text and "from oracle" not in text, f
+
+
+def _cuda_lib_dir():
+    for d in ("/usr/local/cuda/lib64", "/usr/local/cuda/targets/sbsa-linux/lib",
+              "/usr/local/cuda/targets/x86_64-linux/lib"):
+        if os.path.exists(os.path.join(d, "libcudart.so")):
+            return d
+    return None
+
+
+def test_header_is_plain_c_and_links(lib, tmp_path):
+    """include/tv.h compiles as strict C99 and as C++, and a C program that
+    takes every entry point's address links against libtv.so and runs the
+    host-side checks (no device needed)."""
+    import shutil
+    import subprocess
+    cc, cxx = shutil.which("gcc"), shutil.which("g++")
+    cudadir = _cuda_lib_dir()
+    if not cc or not cxx or not cudadir:
+        pytest.skip("no C toolchain or CUDA runtime library")
+    inc = os.path.join(ROOT, "include")
+    src = os.path.join(ROOT, "tests", "c_abi", "use_abi.c")
+    libdir = os.path.dirname(lib._name)
+    exe = str(tmp_path / "use_abi")
+    r = subprocess.run([cc, "-std=c99", "-Wall", "-Wextra", "-Werror", "-pedantic", "-I", inc,
+                        src, "-o", exe, "-L", libdir, "-ltv", f"-Wl,-rpath,{libdir}",
+                        f"-Wl,-rpath-link,{cudadir}", f"-Wl,-rpath,{cudadir}"],
+                       capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    hdr = tmp_path / "hdr.cc"
+    hdr.write_text('#include "tv.h"\nint main() { return tv_version() > 0 ? 0 : 1; }\n')
+    r = subprocess.run([cxx, "-std=c++17", "-Wall", "-Werror", "-fsyntax-only", "-I", inc,
+                        str(hdr)], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    r = subprocess.run([exe], capture_output=True, text=True, timeout=120)
+    assert r.returncode == 0 and r.stdout.strip().endswith("ok"), (r.returncode, r.stdout,
+                                                                   r.stderr)
