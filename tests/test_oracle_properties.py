@@ -27,6 +27,13 @@ def trees(draw, max_nodes=6):
     return parents
 
 
+def depth(parents):
+    d = [0] * len(parents)
+    for i in range(1, len(parents)):
+        d[i] = d[parents[i]] + 1
+    return max(d)
+
+
 @settings(max_examples=60, deadline=None)
 @given(trees(), st.integers(2, 3), st.integers(0, 10 ** 6), st.sampled_from([0.0, 0.3]))
 def test_lossless_on_random_shapes(parents, V, seed, zero_prob):
@@ -36,8 +43,9 @@ def test_lossless_on_random_shapes(parents, V, seed, zero_prob):
     branching = max(parents[1:].count(i) for i in range(len(parents)))
     if branching > V:
         return                                  # more siblings than tokens: no valid tree
-    t = rational_table(V, 3, seed, zero_prob=zero_prob)
-    s = rational_table(V, 3, seed + 1, zero_prob=zero_prob, min_support=branching)
+    L = depth(parents)                          # rows for every prefix up to the leaves
+    t = rational_table(V, L, seed, zero_prob=zero_prob)
+    s = rational_table(V, L, seed + 1, zero_prob=zero_prob, min_support=branching)
     zl, g = z_law(parents, t, s, V)
     tl = target_law(t, V, g)
     assert set(zl) <= set(tl)
@@ -53,8 +61,9 @@ def test_token_level_lossless_on_random_shapes(parents, V, seed):
     branching = max(parents[1:].count(i) for i in range(len(parents)))
     if branching > V:
         return
-    t = rational_table(V, 3, seed)
-    s = rational_table(V, 3, seed + 1, min_support=branching)
+    L = depth(parents)
+    t = rational_table(V, L, seed)
+    s = rational_table(V, L, seed + 1, min_support=branching)
     zl, g = z_law(parents, t, s, V, outcome=tokenlevel.outcome_law)
     tl = target_law(t, V, g)
     assert set(zl) <= set(tl)
