@@ -212,3 +212,32 @@ def test_new_entry_points_argument_errors(tv):
     with pytest.raises(tv.LibraryError):
         v.verify_stats(par, out, lg, dr, 1.0, torch.zeros(4, 9, device="cuda"), st)
     v.close()
+
+
+def test_bench_size_sampled_rows(tv):
+    """The bench's launch: 7808 x 4096 x 128256, 61 row tiles walked in two
+    groups (32 and a tail of 29).  Exact operands, so sampled rows from both
+    groups and the edges of row tiles must equal the oracle bit for bit over
+    every column, with their normalisers."""
+    M, K, V, B, N = 7808, 4096, 128256, 128, 60
+    g = torch.Generator(device="cuda").manual_seed(61)
+    H = (torch.randint(-8, 9, (M, K), generator=g, device="cuda") / 16.0).to(torch.bfloat16)
+    W = (torch.randint(-8, 9, (V, K), generator=g, device="cuda") / 16.0).to(torch.bfloat16)
+    v = tv.Verifier(V, N, B, "bf16", path="persistent")
+    lg, st = v.lm_head(H, W, 0.7)
+    torch.cuda.synchronize()
+    assert v.status() == 0
+    v.close()
+    rows = [0, 1, 127, 128, 2047, 4095, 4096, 4097, 6000, 7679, 7680, 7807]
+    h = H[rows].float().cpu().numpy()
+    got = lg[rows].float().cpu().numpy().astype(np.float64)
+    st = st[rows].cpu().numpy().astype(np.float64)
+    ref = np.empty((len(rows), V))
+    Wc = W.float().cpu().numpy()
+    for v0 in range(0, V, 16384):
+        ref[:, v0:v0 + 16384] = lmhead.logits(h, Wc[v0:v0 + 16384])
+    ref = lmhead.to_bf16(ref)
+    assert np.array_equal(got, ref)
+    m, s = lmhead.row_stats(ref, 0.7)
+    assert np.array_equal(st[:, 0], m)
+    assert np.max(np.abs(st[:, 1] - s) / s) < 1e-5
