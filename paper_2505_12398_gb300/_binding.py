@@ -100,6 +100,15 @@ def _stream_ptr(stream):
     return ctypes.c_void_p(stream.cuda_stream)
 
 
+def _check_out(t, dtype, shape, device):
+    """An output tensor the library writes: its dtype, shape, contiguity and
+    device must be what the call's sizes say (the kernels trust them)."""
+    if t.dtype != dtype or tuple(t.shape) != tuple(shape) or not t.is_contiguous() \
+            or t.device != device:
+        raise ValueError(f"output: expected a contiguous {dtype} {tuple(shape)} tensor on "
+                         f"{device}, got {t.dtype} {tuple(t.shape)} on {t.device}")
+
+
 class Verifier:
     """Owns a ``tv_handle`` (device workspace) for one device and size limits.
 
@@ -173,6 +182,8 @@ class Verifier:
             bonus = torch.empty(B, dtype=torch.int32, device=self.device)
         else:
             path, tau, bonus = out
+            for t, shape in ((path, (B, N)), (tau, (B,)), (bonus, (B,))):
+                _check_out(t, torch.int32, shape, self.device)
         sp = _stream_ptr(stream)
         if debug:
             node_p = torch.empty(B, N + 1, dtype=torch.float32, device=self.device)
@@ -207,6 +218,10 @@ class Verifier:
             row_stats = torch.empty(M, 2, dtype=torch.float32, device=self.device)
         else:
             logits, row_stats = out
+            if logits.numel() != M * self.vocab or row_stats.numel() != 2 * M:
+                raise ValueError("output: logits must hold M x V and row_stats M x 2 values")
+            _check_out(logits, torch.bfloat16, logits.shape, self.device)
+            _check_out(row_stats, torch.float32, row_stats.shape, self.device)
         rc = self.lib.tv_lm_head(self.handle, M, K, _ptr(hidden), _ptr(weight),
                                  float(temperature), _ptr(logits), _ptr(row_stats),
                                  _stream_ptr(stream))
@@ -227,6 +242,7 @@ class Verifier:
                     or t.device != self.device:
                 raise ValueError(f"expected a contiguous {dt} {shape} tensor on {self.device}")
         tokens = torch.empty(B, R, dtype=torch.int32, device=self.device) if out is None else out
+        _check_out(tokens, torch.int32, (B, R), self.device)
         rc = self.lib.tv_draft_children(self.handle, B, R - 1, _ptr(parents), _ptr(drafts),
                                         _ptr(uniforms), _ptr(tokens), _stream_ptr(stream))
         if rc != 0:
@@ -249,6 +265,8 @@ class Verifier:
             bonus = torch.empty(B, dtype=torch.int32, device=self.device)
         else:
             path, tau, bonus = out
+            for t, shape in ((path, (B, N)), (tau, (B,)), (bonus, (B,))):
+                _check_out(t, torch.int32, shape, self.device)
         node_p = torch.empty(B, N + 1, dtype=torch.float32, device=self.device) if debug else None
         stats = torch.empty(B, 5, dtype=torch.int32, device=self.device) if debug else None
         rc = self.lib.tv_verify_batch_stats(

@@ -91,3 +91,16 @@ def test_header_is_plain_c_and_links(lib, tmp_path):
     r = subprocess.run([exe], capture_output=True, text=True, timeout=120)
     assert r.returncode == 0 and r.stdout.strip().endswith("ok"), (r.returncode, r.stdout,
                                                                    r.stderr)
+
+
+def test_binding_checks_output_tensors():
+    """Outputs the kernels write are checked for dtype, shape, contiguity and
+    device before any call (the kernels trust the sizes)."""
+    import torch
+    from paper_2505_12398_gb300._binding import _check_out
+    cpu = torch.device("cpu")
+    _check_out(torch.zeros(2, 3, dtype=torch.int32), torch.int32, (2, 3), cpu)
+    for bad in (torch.zeros(2, 3), torch.zeros(3, 2, dtype=torch.int32),
+                torch.zeros(3, 2, dtype=torch.int32).t()):
+        with pytest.raises(ValueError):
+            _check_out(bad, torch.int32, (2, 3), cpu)
