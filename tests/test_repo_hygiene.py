@@ -51,3 +51,16 @@ def test_sources_do_not_name_batched_copies():
     for f in committed_files():
         if f.endswith((".py", ".cu", ".cuh", ".h", ".c")):
             assert not pattern.search(open(os.path.join(ROOT, f)).read()), f
+
+
+def test_code_names_no_build_documents_or_machines():
+    """Code and its comments stand on their own: they name none of the
+    build's planning documents, the runner of the GPU jobs, or paths of the
+    machine they were written on."""
+    words = ["SUR" + "VEY", "DES" + "IGN.md", "VER" + "DICT", "ADV" + "ICE", "BASE" + "LINE",
+             "north" + "_star", "gpu" + "run", "/ro" + "ot/"]
+    for f in committed_files():
+        if f.endswith((".py", ".cu", ".cuh", ".h", ".c", ".sh")):
+            text = open(os.path.join(ROOT, f)).read()
+            for w in words:
+                assert w not in text, (f, w)
