@@ -3,9 +3,12 @@
 Usage: ``python -m paper_2505_12398_gb300.build`` (or ``build()`` from
 Python).  Each translation unit is compiled in parallel with nvcc, then
 linked into a shared library next to this file.  Rebuilds only when a source
-is newer than the library.
+is newer than the library.  Concurrent callers (e.g. the ranks of a multi-GPU
+run) are serialised by a file lock, and a caller that waited finds the library
+built.
 """
 
+import fcntl
 import os
 import shutil
 import subprocess
@@ -44,10 +47,26 @@ def _stale():
     return any(os.path.getmtime(d) > t for d in deps)
 
 
+def with_build_lock(fn):
+    """Runs fn() holding the build folder's exclusive lock (across processes)."""
+    os.makedirs(BUILD, exist_ok=True)
+    with open(os.path.join(BUILD, ".lock"), "w") as lock:
+        fcntl.flock(lock, fcntl.LOCK_EX)
+        try:
+            return fn()
+        finally:
+            fcntl.flock(lock, fcntl.LOCK_UN)
+
+
 def build(force=False, verbose=False):
     """Compile libtv.so if needed; returns its path."""
     if not force and not _stale():
         return LIB
+    return with_build_lock(lambda: LIB if (not force and not _stale())
+                           else _build(verbose))
+
+
+def _build(verbose):
     nvcc = _nvcc()
     os.makedirs(BUILD, exist_ok=True)
 
