@@ -104,3 +104,15 @@ def test_binding_checks_output_tensors():
                 torch.zeros(3, 2, dtype=torch.int32).t()):
         with pytest.raises(ValueError):
             _check_out(bad, torch.int32, (2, 3), cpu)
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    """Without the compiled library the binding raises; there is no CPU
+    implementation to fall back to."""
+    from paper_2505_12398_gb300 import _binding
+    monkeypatch.setattr(_binding, "_LIB", None)
+    monkeypatch.setattr(_binding, "library_path", lambda: str(tmp_path / "libtv.so"))
+    with pytest.raises(ImportError):
+        _binding.library()
+    with pytest.raises(ImportError):
+        _binding.Verifier(1000, 7, 4, "bf16")
