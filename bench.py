@@ -31,6 +31,11 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
+# The headline: the largest single-GPU throughput configuration, 60-node
+# EAGLE-shaped trees at V = 151936 (bf16), 1024 trees, draft noise 2 (the
+# low-acceptance end of the sweep).  The other pipelines default to the
+# 128-tree, V = 128256 workload.
+DEFAULT_VERIFY = ("sweep60", 1024, 2.0)
 DEFAULT_WORKLOAD = "eagle_v128k"
 
 
@@ -40,7 +45,7 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--workload", default=None)
     ap.add_argument("--batch", type=int, default=None)
     ap.add_argument("--sigma", type=float, default=None)
     ap.add_argument("--seed", type=int, default=0)
@@ -63,7 +68,18 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="rough budget of the CPU-baseline sample")
-    return ap.parse_args()
+    ap.add_argument("--no-extra", action="store_true",
+                    help="skip the other workloads timed after the headline one")
+    ap.add_argument("--extra-steps", type=int, default=20)
+    args = ap.parse_args()
+    if args.workload is None:
+        if args.pipeline == "verify":
+            args.workload = DEFAULT_VERIFY[0]
+            args.batch = DEFAULT_VERIFY[1] if args.batch is None else args.batch
+            args.sigma = DEFAULT_VERIFY[2] if args.sigma is None else args.sigma
+        else:
+            args.workload = DEFAULT_WORKLOAD
+    return args
 
 
 # ------------------------------------------------------ multi-rank ---------
@@ -257,23 +273,44 @@ def time_oracle(sample_dir, n_trees, temperature, pool, reps=1, method="traversa
 
 # ---------------------------------------------------------- helpers ---------
 
-def algorithmic_bytes(stats, tau, V, logit_bytes):
-    """Bytes of target logits and draft probabilities the verification has to
-    read, per tree: one target row for every normaliser computed (stats column
-    4), one target row and one draft row for every S-computation of
-    Eqs. (1)/(3) (column 1: each pass depends on the distribution the previous
-    one left), and one row (target only for an original leaf, target and draft
-    for a residual) for the bonus draw.  Returns (normaliser bytes, pass and
-    bonus bytes)."""
+def algorithmic_bytes(stats, tau, parents, V, logit_bytes):
+    """Bytes of target logits and draft probabilities per step, three ways,
+    from the debug entry point's per-tree counts (stats columns: tests,
+    S-passes, distinct nodes with a pass R, bonus from an original leaf,
+    rows normalised):
+
+    * ``unique``: every row the call needed, each counted once -- the target
+      rows it normalised, the draft rows of the R nodes with passes (their
+      target rows are among the normalised ones) and, when the bonus came
+      from an original leaf, that leaf's target row.  The roofline's bytes.
+    * ``s8d``: the count A = |I| V s_l + R V 4 + [leaf] V s_l under the
+      eager initialisation of Algorithm 3 (every internal row normalised).
+    * ``reread``: what the passes stream, re-reads included: every S-pass
+      reads its target and draft rows again (the residual it sums depends on
+      the previous pass), the bonus reads one row (target only at a leaf).
+    Invalid trees count nothing."""
     import torch
-    valid = tau >= 0
-    norm = stats[:, 4].to(torch.int64)
-    passes = stats[:, 1].to(torch.int64)
-    leaf = stats[:, 3].to(torch.int64)
-    row_bytes = norm * V * logit_bytes
-    bonus = torch.where(leaf > 0, V * logit_bytes, V * (logit_bytes + 4)) * valid.to(torch.int64)
-    other = passes * V * (logit_bytes + 4) + bonus
-    return int(row_bytes.sum()), int(other.sum())
+    valid = (tau >= 0).to(torch.int64)
+    norm = stats[:, 4].to(torch.int64) * valid
+    passes = stats[:, 1].to(torch.int64) * valid
+    R = stats[:, 2].to(torch.int64) * valid
+    leaf = stats[:, 3].to(torch.int64) * valid
+    par = parents.to(torch.int64)
+    n_int = torch.zeros_like(par)
+    n_int.scatter_(1, par[:, 1:].clamp(min=0), 1)
+    internal = n_int.sum(1) * valid
+    lb = logit_bytes
+    unique = norm * V * lb + R * V * 4 + leaf * V * lb
+    s8d = internal * V * lb + R * V * 4 + leaf * V * lb
+    bonus = torch.where(leaf > 0, V * lb, V * (lb + 4)) * valid
+    reread = norm * V * lb + passes * V * (lb + 4) + bonus
+    n = max(int(valid.sum()), 1)
+    return {"unique": int(unique.sum()), "s8d": int(s8d.sum()), "reread": int(reread.sum()),
+            "normaliser": int((norm * V * lb).sum()),
+            "R_per_tree": float(R.sum()) / n, "passes_per_tree": float(passes.sum()) / n,
+            "rows_normalised_per_tree": float(norm.sum()) / n,
+            "internal_rows_per_tree": float(internal.sum()) / n,
+            "leaf_bonus_frac": float(leaf.sum()) / n}
 
 
 def main():
@@ -317,14 +354,22 @@ def main():
 
     # decisions are a deterministic function of the inputs: one instrumented
     # call gives the rows each tree needs (algorithmic bytes) and tau
-    _, tau_d, _, _, stats = v.verify(inp.parents, inp.tokens, inp.logits, inp.draft_probs,
-                                     inp.temperature, inp.uniforms, debug=True)
+    _, tau_d, _, _, stats, margin = v.verify(inp.parents, inp.tokens, inp.logits,
+                                             inp.draft_probs, inp.temperature, inp.uniforms,
+                                             debug=True, margins=True)
     torch.cuda.synchronize(dev)
-    row_bytes, trav_bytes = algorithmic_bytes(stats, tau_d, V, lb)
+    ab = algorithmic_bytes(stats, tau_d, inp.parents, V, lb)
+    # near-ties as the GPU itself reports them (decision margin below 1e-5)
+    near_ties = {"tests": int((margin[:, 0] < 1e-5).sum()),
+                 "bonus": int((margin[:, 1] < 1e-5).sum()),
+                 "trees": int(((margin[:, 0] < 1e-5) | (margin[:, 1] < 1e-5)).sum()),
+                 "invalid_trees": int((tau_d < 0).sum())}
+    row_bytes = ab["normaliser"]
+    trav_bytes = ab["reread"] - row_bytes
     path_code, cluster, warps, stages = v.launch_shape(B, N)
-    a_bytes = row_bytes + trav_bytes
+    a_bytes = ab["unique"]
     mean_tau1 = float(tau_d.float().mean()) + 1.0
-    passes_per_tree = float(stats[:, 1].float().mean())
+    passes_per_tree = ab["passes_per_tree"]
 
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     out = (torch.empty(B, N, dtype=torch.int32, device=dev),
@@ -371,8 +416,13 @@ def main():
     # end to end through the public API from pinned host buffers
     e2e = None
     if not args.no_e2e:
-        hp = [x.cpu().pin_memory() for x in (inp.parents, inp.tokens, inp.logits,
-                                              inp.draft_probs, inp.uniforms)]
+        # pinned host copies made directly (no pageable intermediate: the
+        # headline batch holds tens of GB)
+        hp = []
+        for x in (inp.parents, inp.tokens, inp.logits, inp.draft_probs, inp.uniforms):
+            h = torch.empty(x.shape, dtype=x.dtype, pin_memory=True)
+            h.copy_(x)
+            hp.append(h)
         hout = (torch.empty(B, N, dtype=torch.int32).pin_memory(),
                 torch.empty(B, dtype=torch.int32).pin_memory(),
                 torch.empty(B, dtype=torch.int32).pin_memory())
@@ -402,6 +452,16 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(inp, args, B)
 
+    # free the headline batch, then time the other configurations
+    v.close()
+    del inp, out, flush
+    torch.cuda.empty_cache()
+    extras = None
+    if world == 1 and not args.no_extra and args.method == "traversal":
+        extras = [measure_extra(tv, n, b, sg, args, dev) for n, b, sg in EXTRA_CONFIGS
+                  if (n, b, sg if sg is not None else get_workload(n).sigma) !=
+                  (w.name, B, w.sigma)]
+
     peak, peak_kind = measured_peaks()
     ph = [sum(p[i] for p in phase) / len(phase) for i in range(3)]
     if path_code == 0:
@@ -422,6 +482,21 @@ def main():
     trees_s = whole_job_rate(B, world, args.steps, total_ms_max)
     step_gbs = a_bytes / (ms_step / 1e3) / 1e9
     dom_gbs = kbytes[dom] / (ph[dom] / 1e3) / 1e9 if ph[dom] > 0 else 0.0
+    dom_s = ph[dom] / 1e3 if ph[dom] > 0 else float("inf")
+
+    def frac(nbytes):
+        return round(nbytes / dom_s / 1e9 / peak, 4)
+
+    roof = {"bound": "hbm", "kernel": names[dom], "achieved": round(dom_gbs, 2),
+            "peak": peak, "unit": "GB/s", "frac": round(dom_gbs / peak, 4),
+            "peak_kind": peak_kind, "bytes": "unique rows needed, each once",
+            "bytes_per_launch": kbytes[dom], "traffic": traffic}
+    if path_code != 0:
+        roof["frac_reread_inclusive"] = frac(ab["reread"])
+        roof["frac_eager_A"] = frac(ab["s8d"])
+        if traffic:
+            roof["dram_frac"] = frac(traffic)
+            roof["traffic_over_unique"] = round(traffic / max(ab["unique"], 1), 4)
     line = {
         "metric": "verified trees/sec and logit GB/s (fraction of HBM peak) at batch B, "
                   "vocab V, 1 GB300",
@@ -438,7 +513,6 @@ def main():
         "data": "synthetic (seeded logits with Zipf rank prior, noisy-drafter probabilities, "
                 "EAGLE-shaped draft trees sampled without replacement)",
         "config": {"workload": w.name, "batch": B, "vocab": V, "nodes": N, "method": args.method,
-                   "normalised_rows_per_tree": round(row_bytes / (V * lb) / B, 3) if B else 0,
                    "logit_dtype": "bf16" if lb == 2 else "fp32",
                    "temperature": w.temperature, "sigma": w.sigma, "seed": args.seed,
                    "l2": "flushed by a 256 MiB write before every timed step (untimed)",
@@ -448,27 +522,91 @@ def main():
                    "ctas_per_tree": cluster, "consumer_warps": warps, "ring_stages": stages},
         "verified_logit_gbps": round(step_gbs, 2),
         "hbm_frac_step": round(step_gbs / peak, 4),
-        "algorithmic_bytes_per_step": a_bytes,
+        "bytes_per_step": {"unique": ab["unique"], "eager_A": ab["s8d"],
+                           "reread_inclusive": ab["reread"]},
+        "per_tree": {k: round(ab[k], 4) for k in ("R_per_tree", "passes_per_tree",
+                                                  "rows_normalised_per_tree",
+                                                  "internal_rows_per_tree",
+                                                  "leaf_bonus_frac")},
         "mean_accept_len_tau_plus_1": round(mean_tau1, 4),
-        "rejection_passes_per_tree": round(passes_per_tree, 3),
+        "near_ties_margin_below_1e-5": near_ties,
         "phase_ms": {names[i]: round(ph[i], 6) for i in range(3) if names[i] != "-"},
-        "roofline": {"bound": "hbm", "kernel": names[dom], "achieved": round(dom_gbs, 2),
-                     "peak": peak, "unit": "GB/s", "frac": round(dom_gbs / peak, 4),
-                     "peak_kind": peak_kind, "bytes_per_launch": kbytes[dom],
-                     "traffic": traffic},
+        "roofline": roof,
         "roofline_step": {"bound": "hbm", "achieved": round(step_gbs, 2), "peak": peak,
                           "unit": "GB/s", "frac": round(step_gbs / peak, 4)},
         "e2e": e2e,
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clocks,
         "cpu_baseline": cpu,
+        "other_configs": extras,
         "wall_s_timed_region": round(wall, 3),
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
-    v.close()
     if world > 1:
         dist.destroy_process_group()
+
+
+# The other configurations, timed after the headline one (one GPU, rank 0):
+# 64 EAGLE-shaped trees at V = 32000, 128 at V = 128256 (T = 0.7), and the other
+# corners of the V = 151936 throughput sweep.
+EXTRA_CONFIGS = (("eagle_v32k", 64, None), ("eagle_v128k", 128, None), ("sweep60", 1024, 0.5),
+                 ("sweep26", 1024, 2.0), ("sweep120", 1024, 2.0))
+
+
+def measure_extra(tv, name, batch, sigma, args, dev):
+    """Device time of one more workload on a fresh handle: warm-up, then
+    args.extra_steps timed calls (L2 flushed before each), with the same byte
+    counts as the headline."""
+    import torch
+    from workloads.synth import get_workload, make_inputs
+    w = get_workload(name, batch=batch, sigma=sigma)
+    inp = make_inputs(w, seed=args.seed, device=dev)
+    B, R = inp.parents.shape
+    N, V = R - 1, w.vocab
+    lb = 2 if inp.logits.dtype == torch.bfloat16 else 4
+    v = tv.Verifier(V, N, B, "bf16" if lb == 2 else "fp32", device=dev.index, path=args.path,
+                    method=args.method)
+    stream = torch.cuda.current_stream(dev)
+    _, tau_d, _, _, stats = v.verify(inp.parents, inp.tokens, inp.logits, inp.draft_probs,
+                                     inp.temperature, inp.uniforms, debug=True)
+    torch.cuda.synchronize(dev)
+    ab = algorithmic_bytes(stats, tau_d, inp.parents, V, lb)
+    out = (torch.empty(B, N, dtype=torch.int32, device=dev),
+           torch.empty(B, dtype=torch.int32, device=dev),
+           torch.empty(B, dtype=torch.int32, device=dev))
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    times = []
+    for k in range(max(3, args.warmup) + args.extra_steps):
+        flush.zero_()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        v.verify(inp.parents, inp.tokens, inp.logits, inp.draft_probs, inp.temperature,
+                 inp.uniforms, out=out, stream=stream)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        if k >= max(3, args.warmup):
+            times.append(e0.elapsed_time(e1))
+    status = v.status()
+    v.close()
+    del inp, flush, out
+    torch.cuda.empty_cache()
+    peak, _ = measured_peaks()
+    ms = sum(times) / len(times)
+    sec = ms / 1e3
+    return {"workload": name, "batch": B, "vocab": V, "nodes": N, "sigma": w.sigma,
+            "temperature": w.temperature, "steps": len(times), "ms_per_step": round(ms, 6),
+            "trees_per_s": round(B / sec, 1),
+            "frac_unique": round(ab["unique"] / sec / 1e9 / peak, 4),
+            "frac_reread_inclusive": round(ab["reread"] / sec / 1e9 / peak, 4),
+            "frac_eager_A": round(ab["s8d"] / sec / 1e9 / peak, 4),
+            "bytes_per_step": {"unique": ab["unique"], "eager_A": ab["s8d"],
+                               "reread_inclusive": ab["reread"]},
+            "per_tree": {k: round(ab[k], 4) for k in ("R_per_tree", "passes_per_tree",
+                                                      "rows_normalised_per_tree",
+                                                      "internal_rows_per_tree")},
+            "status": int(status)}
 
 
 def cpu_baseline(inp, args, B):
@@ -678,7 +816,8 @@ def main_lmhead(args, world, rank, local_rank):
     torch.cuda.synchronize(dev)
     if v.status() & ~16:
         raise RuntimeError(f"device status {tv.status_names(v.status())}")
-    _, trav_bytes = algorithmic_bytes(stats, tau_d, V, 2)
+    ab = algorithmic_bytes(stats, tau_d, inp.parents, V, 2)
+    trav_bytes = ab["reread"] - ab["normaliser"]
     mean_tau1 = float(tau_d.float().mean()) + 1.0
 
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)

@@ -182,14 +182,26 @@ int tv_verify_batch(tv_handle* h, int B, int N, const int32_t* parents,
  *               depends on the kernel path (the three-kernel path normalises
  *               every internal row, the single-kernel paths only the rows the
  *               traversal reaches).
- * Either pointer may be NULL.  Other arguments and errors as tv_verify_batch.
+ *   out_margin  [B][2] fp32 (device): the tree's decision margins, computed
+ *               on the GPU, for counting near-ties on batches no oracle sees.
+ *               [b][0] = min over the tree's tests of |eta - p| (Algorithm 3's
+ *               strict eta < p test, p as recorded in out_node_p); +inf if
+ *               the tree had no test.  [b][1] = the bonus draw's margin
+ *               min(u W - CDF(Y - 1), CDF(Y) - u W) / W from the kernel's own
+ *               float32 cumulative sums (0 when rounding put u W past the
+ *               total).  A decision whose margin is below about 1e-6 may
+ *               differ from an exact float64 evaluation.  NaN for an
+ *               invalid tree.
+ * Any of the three pointers may be NULL.  Other arguments and errors as
+ * tv_verify_batch.
  */
 int tv_verify_batch_debug(tv_handle* h, int B, int N, const int32_t* parents,
                           const int32_t* draft_tokens, const void* target_logits,
                           const float* draft_probs, float temperature,
                           const float* uniforms, int32_t* out_accepted_path,
                           int32_t* out_accept_len, int32_t* out_bonus_token,
-                          float* out_node_p, int32_t* out_stats, void* cuda_stream);
+                          float* out_node_p, int32_t* out_stats, float* out_margin,
+                          void* cuda_stream);
 
 /*
  * tv_verify_batch_host -- the same verification from HOST buffers: copies the
@@ -338,9 +350,11 @@ int tv_launch_shape(tv_handle* h, int B, int N, int* path, int* cluster, int* wa
 
 /*
  * tv_verify_batch_noalloc -- the same verification for callers that cannot
- * allocate device memory (inside a CUDA-graph capture they do not own, under
- * a memory pool that forbids new allocations, or where another allocator owns
- * the device).  The paper has no counterpart: this is a deployment entry point.
+ * allocate device memory: a serving process whose allocator reserved the
+ * device's memory up front and forbids new allocations once it has warmed
+ * up, or an embedding in another runtime that owns every byte of the device.
+ * tv_create allocates a handle's workspace, so such callers cannot use it.
+ * The paper has no counterpart: this is a deployment entry point.
  *
  * Needs no handle and allocates nothing: its scratch (internal-row list, row
  * statistics, status word) is one fixed array of static device memory in the
@@ -352,6 +366,11 @@ int tv_launch_shape(tv_handle* h, int B, int N, int* path, int* cluster, int* wa
  * call before any stream capture.  All calls share the array: each clears
  * what must start at zero, but calls whose work overlaps on the GPU race on it
  * and must not be issued.
+ *
+ * No TV_STATUS_* word is reported on this path: the status word lives in the
+ * shared array and no call returns it.  An invalid tree (BAD_TREE, BAD_TOKEN,
+ * DUP_SIBLING, ZERO_DRAFT, BAD_ROW) shows only as accept_len = -1, bonus = -1
+ * and a path of -1 for that tree; the informational DEGENERATE bit is lost.
  *   device      : CUDA device ordinal (0..63) the pointers belong to.
  *   vocab, logit_dtype : as in tv_create.
  *   the rest    : as in tv_verify_batch (device pointers, caller-owned).

@@ -124,11 +124,13 @@ def validate_tree(parents, tokens, vocab, allow_duplicate_siblings=False):
 def _condition(p, mb, ms, S):
     """Instrumentation only: relative sensitivity of S to relative
     perturbations of M_b, sum over the positive part of p M_b(x), divided by
-    S (inf when S = 0).  A float computation of S whose M_b values carry a
-    relative error e has a relative error of about e times this number."""
+    S.  A float computation of S whose M_b values carry a relative error e
+    has a relative error of about e times this number."""
     pos = (p * mb - ms) > 0
     if not S > 0:
-        return float("inf")
+        # the 0/0 of Eqs. (1)/(3) is resolved exactly (p' = 0 removes the
+        # node, p = 1 keeps its row), so no rounding error flows from it
+        return 1.0
     return float((p * mb)[pos].sum() / S)
 
 
@@ -180,6 +182,7 @@ class TraversalState:
         # nodes removed with rate 0, and the bonus row fetched for a leaf
         self.passes = [0] * n
         self.kappa = []         # condition number of each S (instrumentation)
+        self.kappa_S = []       # the S each kappa entry belongs to (instrumentation)
         self.degenerate = 0
         self.pruned = []
         self.leaf_rows_read = set()
@@ -252,6 +255,7 @@ class TraversalState:
         S = residual_mass(p, mb, ms)
         self.passes[i] += 1
         self.kappa.append(_condition(p, mb, ms, S))
+        self.kappa_S.append(float(S))
         if S > 0:
             new_mb = residual_target(p, mb, ms, S)
             new_p = updated_rate(p, S)
@@ -261,6 +265,7 @@ class TraversalState:
                 if self.alive[d]:
                     x = self.tokens[d]
                     self.kappa.append(self.kappa[-1] + _cancellation(p * mb[x], ms[x]))
+                    self.kappa_S.append(float(S))
         else:
             self.degenerate += 1
             new_mb = mb

@@ -72,6 +72,7 @@ def verify_tree(parents, tokens, logits, draft_probs, temperature, uniforms, kee
     node_p = np.full(n, np.nan)
     tests = []
     kappa_at_test = []
+    S_at_test = []
     while True:
         leaf = st.first_leaf()
         if leaf == 0:
@@ -81,6 +82,7 @@ def verify_tree(parents, tokens, logits, draft_probs, temperature, uniforms, kee
         node_p[leaf] = p
         tests.append((leaf, float(u[leaf]), p))
         kappa_at_test.append(max(st.kappa, default=1.0))
+        S_at_test.append(st.kappa_S[int(np.argmax(st.kappa))] if st.kappa else float("nan"))
         if u[leaf] < p:
             accepted = leaf
             break
@@ -100,6 +102,7 @@ def verify_tree(parents, tokens, logits, draft_probs, temperature, uniforms, kee
         "node_p": node_p,
         "tests": tests,
         "kappa_at_test": kappa_at_test,
+        "S_at_test": S_at_test,
         "test_margin": min((abs(uu - pp) for _, uu, pp in tests), default=np.inf),
         "bonus_margin": y_margin,
         "bonus_total": W,

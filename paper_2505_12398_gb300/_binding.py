@@ -46,7 +46,8 @@ _F = ctypes.c_float
 _SIGS = {
     "tv_create": (_I, [ctypes.POINTER(_P), _I, _I, _I, _I, _I, ctypes.c_uint]),
     "tv_verify_batch": (_I, [_P, _I, _I, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P]),
-    "tv_verify_batch_debug": (_I, [_P, _I, _I, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P, _P, _P]),
+    "tv_verify_batch_debug": (_I, [_P, _I, _I, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P, _P, _P,
+                                   _P]),
     "tv_verify_batch_host": (_I, [_P, _I, _I, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P]),
     "tv_verify_batch_stats": (_I, [_P, _I, _I, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P, _P, _P,
                                    _P]),
@@ -170,9 +171,10 @@ class Verifier:
         return B, N
 
     def verify(self, parents, tokens, logits, drafts, temperature, uniforms,
-               out=None, stream=None, debug=False):
+               out=None, stream=None, debug=False, margins=False):
         """Returns (path [B,N] int32, tau [B] int32, bonus [B] int32) as CUDA
-        tensors, plus (node_p [B,N+1] f32, stats [B,4] int32) when ``debug``.
+        tensors, plus (node_p [B,N+1] f32, stats [B,5] int32) when ``debug``,
+        plus margins [B,2] f32 (test, bonus) when ``margins`` too.
         Asynchronous on ``stream`` (default: torch's current stream)."""
         import torch
         B, N = self._check(parents, tokens, logits, drafts, uniforms)
@@ -188,12 +190,15 @@ class Verifier:
         if debug:
             node_p = torch.empty(B, N + 1, dtype=torch.float32, device=self.device)
             stats = torch.empty(B, 5, dtype=torch.int32, device=self.device)
+            margin = torch.empty(B, 2, dtype=torch.float32, device=self.device)
             rc = self.lib.tv_verify_batch_debug(
                 self.handle, B, N, _ptr(parents), _ptr(tokens), _ptr(logits), _ptr(drafts),
                 float(temperature), _ptr(uniforms), _ptr(path), _ptr(tau), _ptr(bonus),
-                _ptr(node_p), _ptr(stats), sp)
+                _ptr(node_p), _ptr(stats), _ptr(margin), sp)
             if rc != 0:
                 raise LibraryError("tv_verify_batch_debug", rc, self.lib)
+            if margins:
+                return path, tau, bonus, node_p, stats, margin
             return path, tau, bonus, node_p, stats
         rc = self.lib.tv_verify_batch(
             self.handle, B, N, _ptr(parents), _ptr(tokens), _ptr(logits), _ptr(drafts),

@@ -203,7 +203,7 @@ int verify_impl(tv_handle* h, int B, int N, const int32_t* parents, const int32_
                 const void* logits, const float* drafts, float temperature,
                 const float* uniforms, int32_t* out_path, int32_t* out_len, int32_t* out_bonus,
                 float* out_node_p, int32_t* out_stats, void* stream,
-                const float2* row_stats = nullptr) {
+                const float2* row_stats = nullptr, float* out_margin = nullptr) {
   int rc = check_call(h, B, N, parents, tokens, logits, drafts, temperature, uniforms,
                       out_path, out_len, out_bonus);
   if (rc != TV_OK || B == 0) return rc;
@@ -228,6 +228,7 @@ int verify_impl(tv_handle* h, int B, int N, const int32_t* parents, const int32_
   a.out_bonus = out_bonus;
   a.out_node_p = out_node_p;
   a.out_stats = out_stats;
+  a.out_margin = out_margin;
   a.status = h->status;
   a.token_level = (h->flags & TV_FLAG_TOKEN_LEVEL) ? 1 : 0;
   a.row_stats = row_stats;
@@ -372,11 +373,12 @@ int tv_verify_batch_debug(tv_handle* h, int B, int N, const int32_t* parents,
                           const float* draft_probs, float temperature,
                           const float* uniforms, int32_t* out_accepted_path,
                           int32_t* out_accept_len, int32_t* out_bonus_token,
-                          float* out_node_p, int32_t* out_stats, void* cuda_stream) {
+                          float* out_node_p, int32_t* out_stats, float* out_margin,
+                          void* cuda_stream) {
   NvtxRange range("tv_verify_batch_debug");
   return verify_impl(h, B, N, parents, draft_tokens, target_logits, draft_probs, temperature,
                      uniforms, out_accepted_path, out_accept_len, out_bonus_token, out_node_p,
-                     out_stats, cuda_stream);
+                     out_stats, cuda_stream, nullptr, out_margin);
 }
 
 int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,

@@ -43,6 +43,7 @@ struct Ctl {
   int accepted;        // accepted node (-1: invalid tree)
   float S;             // result of the last pass
   int bonus_y;
+  float bmargin;       // margin of the bonus draw (out_margin[b][1])
   // serial control state (thread 0)
   int node;
   int pending;         // child whose rejection the running pass serves

@@ -229,4 +229,17 @@ __device__ __forceinline__ float warp_max(float v) {
   return v;
 }
 
+// The smallest |eta - p| over the tree's tests: every node with a positive
+// recorded rate (dbgp, the rate at its test; removals at rate 0 record 0 and
+// untested nodes NaN) was tested with its own uniform u[i].  +inf without a
+// test.  One thread; only for the debug output.
+__device__ inline float test_margin_serial(const float* dbgp, const float* u, int R) {
+  float m = __int_as_float(0x7f800000);
+  for (int i = 1; i < R; ++i) {
+    const float p = dbgp[i];
+    if (p > 0.f) m = fminf(m, (float)fabs((double)u[i] - (double)p));
+  }
+  return m;
+}
+
 }  // namespace tvk

@@ -73,7 +73,8 @@ constexpr int kItemNop = 6;         // FlowItem::kind of a reserved slot that ca
 struct ItemSlot {
   int b, node, row, slice;
   int kind, slice_len, nmask, pad0;
-  float alpha1, beta, rowmax, pad1;
+  float alpha1, beta, rowmax;
+  int par;                 // parity of the job's sequence number (its partials buffer)
 };
 
 struct StageMeta {
@@ -89,7 +90,16 @@ struct Shared {
   Job fjob;                          // a job posted from `ahead`
   float2 pbuf[kPBuf];                // the own job's partials, as read by the poll
   int jkind, jrows, jK, jslice, outstanding;
+  int jseq;                          // sequence number of the own tree's current job
 };
+
+// Partial of (tree b, job parity par, row r of the job, slice k).  Jobs
+// alternate between two buffers, so a job's slices may be reset and written
+// while the previous job's partials are still being read.
+__device__ __forceinline__ unsigned long long* part_at(const FlowArgs& f, int b, int par, int r,
+                                                       int k) {
+  return f.part + (((size_t)b * 2 + par) * f.R + r) * f.Kmax + k;
+}
 
 __device__ __forceinline__ unsigned ld_relaxed_u32(const unsigned* p) {
   unsigned v;
@@ -247,6 +257,7 @@ __device__ void fetcher_role(const TravArgs& a, const FlowArgs& f, const Smem& m
         it.kind = w[1].x; it.slice_len = w[1].y; it.nmask = w[1].z;
         it.alpha1 = __int_as_float(w[2].x); it.beta = __int_as_float(w[2].y);
         it.rowmax = __int_as_float(w[2].z);
+        it.par = w[2].w;
         int* mt = m.mtok + slot * R;
         float* mv = m.mval + slot * R;
         const int ni = min(w[1].z, kFlowInlineMask);
@@ -353,7 +364,7 @@ __device__ void consumer_role(const TravArgs& a, const FlowArgs& f, const Smem& 
   int stage = 0, phase = 0;
   unsigned red_phase = 0u;   // parity bit per stage of red_bar (warp 0 waits on it)
   // the slice in progress
-  int kind = 0, b = 0, row_idx = 0, slice = 0, nmask = 0, slot = 0, x0 = 0, x1 = 0;
+  int kind = 0, b = 0, row_idx = 0, slice = 0, nmask = 0, slot = 0, x0 = 0, x1 = 0, par = 0;
   float alpha1 = 0.f, beta = 0.f, rowmax = 0.f;
   float m_run = TV_NEG_INF;
   Comp acc;
@@ -368,6 +379,7 @@ __device__ void consumer_role(const TravArgs& a, const FlowArgs& f, const Smem& 
     if (meta.flags & kStageFirst) {
       const ItemSlot& it = m.sh->slots[meta.slot];
       kind = it.kind; b = it.b; row_idx = it.row; slice = it.slice; nmask = it.nmask;
+      par = it.par;
       alpha1 = it.alpha1; beta = it.beta; rowmax = it.rowmax;
       slot = meta.slot;
       x0 = slice * it.slice_len;
@@ -607,7 +619,7 @@ __device__ void consumer_role(const TravArgs& a, const FlowArgs& f, const Smem& 
           fence_gpu();   // the tiles before the partial that announces them
         }
         if (lane == 0) {
-          st_relaxed_u64(f.part + ((size_t)b * R + row_idx) * f.Kmax + slice, pack_part(px, py));
+          st_relaxed_u64(part_at(f, b, par, row_idx, slice), pack_part(px, py));
           mbar_arrive(&m.empty_bar[stage]);   // only now may the stage (and red[stage]) be reused
         }
       } else if (lane == 0) {
@@ -682,7 +694,8 @@ __device__ __forceinline__ void reserve_next(const FlowArgs& f, int V, int B, in
 // use the slots reserved in `spec`; otherwise those become "no work" items.
 __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const FlowArgs& f,
                          int b, int V, int lane, unsigned done, Reserve spec, const Job& j,
-                         const int* mask_tok, const float* mask_val) {
+                         const int* mask_tok, const float* mask_val, int seq) {
+  const int par = seq & 1;
   const bool stats = (j.kind == kJobStats);
   const int n_rows = stats ? j.n_rows : 1;
   const bool use_spec = spec.n > 0 && j.kind == kJobPass;
@@ -698,7 +711,7 @@ __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const
   // the job's partial slots start as "not yet"
   for (int q = lane; q < n; q += 32) {
     const int r = q / K;
-    __stcg(f.part + ((size_t)b * R + r) * f.Kmax + (q - r * K), kNoPart);
+    __stcg(part_at(f, b, par, r, q - r * K), kNoPart);
   }
   unsigned base = spec.base;
   if (!use_spec) {
@@ -715,7 +728,7 @@ __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const
   if (spec.n > 0 && !use_spec) nop_bodies(f, spec.base, spec.n, lane);
   const int4 w1 = make_int4(j.kind, slice, nmask, 0);
   const int4 w2 = make_int4(__float_as_int(j.alpha1), __float_as_int(j.beta),
-                            __float_as_int(j.rowmax), 0);
+                            __float_as_int(j.rowmax), par);
   int tk[kFlowInlineMask];
   float vk[kFlowInlineMask];
 #pragma unroll
@@ -756,6 +769,7 @@ __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const
     sh.jrows = n_rows;
     sh.jK = K;
     sh.jslice = slice;
+    sh.jseq = seq;
   }
 }
 
@@ -768,6 +782,7 @@ __device__ void owner_new_tree(const TravArgs& a, const TreeSmem& s, Shared& sh,
   const typename L::elem* logits = reinterpret_cast<const typename L::elem*>(a.logits);
   if (lane == 0) {
     sh.outstanding = 0;
+    sh.jseq = -1;
     sh.ahead.ok = 0;
     Ctl& c = sh.ctl;
     c.bad = 0u;
@@ -876,7 +891,7 @@ __device__ void owner_combine(const TravArgs& a, const FlowArgs& f, const TreeSm
   const bool in_smem = sh.outstanding <= kPBuf;
   auto part_of = [&](int r, int k) -> float2 {
     return in_smem ? sh.pbuf[r * K + k]
-                   : unpack_part(__ldcg(f.part + (row0 + r) * f.Kmax + k));
+                   : unpack_part(__ldcg(part_at(f, b, sh.jseq & 1, r, k)));
   };
   if (sh.jkind == kJobStats) {
     // the rows' normalisers from their slices, one lane per row ...
@@ -1056,6 +1071,19 @@ __device__ void owner_combine(const TravArgs& a, const FlowArgs& f, const TreeSm
 #pragma unroll
     for (int e = 7; e >= 0; --e) if (lt < lbase + pre[e]) found = e;
     const unsigned hit = __ballot_sync(0xffffffffu, found < 8);
+    if (a.out_margin) {
+      // the draw's margin (kernel sums), in the crossing slice's units, then
+      // relative to the total
+      float clo = lbase, chi = lbase;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        if (e == found) chi = lbase + pre[e];
+        if (e + 1 == found) clo = lbase + pre[e];
+      }
+      const float my_margin = fminf(lt - clo, chi - lt) * scale / W;
+      const float bm = hit ? __shfl_sync(0xffffffffu, my_margin, __ffs(hit) - 1) : 0.f;
+      if (lane == 0) sh.ctl.bmargin = bm;
+    }
     int yy;
     if (hit) {
       const int l = __ffs(hit) - 1;
@@ -1083,7 +1111,7 @@ __device__ void owner_combine(const TravArgs& a, const FlowArgs& f, const TreeSm
 // Writes tree b's outputs; true if it was the last tree of the call.
 template <bool kGiven>
 __device__ bool owner_finish(const TravArgs& a, const FlowArgs& f, const TreeSmem& s,
-                             Shared& sh, int b, int lane) {
+                             Shared& sh, const float* u, int b, int lane) {
   const int R = a.N + 1, N = a.N;
   const size_t row0 = (size_t)b * R;
   const bool ok = (sh.ctl.bad & (15u | 32u | 64u)) == 0u;
@@ -1116,6 +1144,11 @@ __device__ bool owner_finish(const TravArgs& a, const FlowArgs& f, const TreeSme
       o[2] = ok ? distinct : 0;
       o[3] = (acc_node >= 0 && s.first[acc_node] < 0) ? 1 : 0;
       o[4] = (ok && !kGiven) ? normalised : 0;   // rows this call streamed
+    }
+    if (a.out_margin) {
+      const float nan = __int_as_float(0x7fc00000);
+      a.out_margin[2 * (size_t)b] = acc_node >= 0 ? test_margin_serial(s.dbgp, u, R) : nan;
+      a.out_margin[2 * (size_t)b + 1] = acc_node >= 0 ? sh.ctl.bmargin : nan;
     }
     if (sh.ctl.bad) atomicOr(a.status, sh.ctl.bad);
     f.finished[b] = (unsigned)f.epoch;
@@ -1155,7 +1188,7 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
       for (int q = lane; q < nout; q += 32) {
         const int r = q / K;
         const unsigned long long v =
-            ld_relaxed_u64(f.part + ((size_t)my_tree * R + r) * f.Kmax + (q - r * K));
+            ld_relaxed_u64(part_at(f, my_tree, sh.jseq & 1, r, q - r * K));
         if (v == kNoPart) all = false;
         else if (q < kPBuf) sh.pbuf[q] = unpack_part(v);
       }
@@ -1236,13 +1269,13 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
           __syncwarp();
           if (post_first) {
             post_job(s, sh, a, f, my_tree, V, lane, __shfl_sync(0xffffffffu, done_est, 0),
-                     spec, sh.fjob, m.mtok2, s.mask_val);
+                     spec, sh.fjob, m.mtok2, s.mask_val, sh.jseq + 1);
             if (lane == 0) control_step_ahead(s, sh.ctl, sh.ahead, accept != 0);
           } else {
             if (lane == 0) control_step_ahead(s, sh.ctl, sh.ahead, accept != 0);
             __syncwarp();
             post_job(s, sh, a, f, my_tree, V, lane, __shfl_sync(0xffffffffu, done_est, 0),
-                     spec, sh.ctl.job, s.mask_tok, s.mask_val);
+                     spec, sh.ctl.job, s.mask_tok, s.mask_val, sh.jseq + 1);
           }
           spec.n = 0;
           if (lane == 0) {
@@ -1261,7 +1294,7 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
     if (sh.ctl.job.kind == kJobDone) {
       if (spec.n > 0) post_nops(a, f, spec, lane);   // before the tree counts as done
       spec.n = 0;
-      const bool last = owner_finish<kGiven>(a, f, s, sh, my_tree, lane);
+      const bool last = owner_finish<kGiven>(a, f, s, sh, m.u, my_tree, lane);
       my_tree = -1;
       if (last) {
         // every tree is done: the tickets now held (slots from the tail up to
@@ -1279,7 +1312,7 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
       }
     } else {
       post_job(s, sh, a, f, my_tree, V, lane, __shfl_sync(0xffffffffu, done_est, 0), spec,
-               sh.ctl.job, s.mask_tok, s.mask_val);
+               sh.ctl.job, s.mask_tok, s.mask_val, sh.jseq + 1);
       spec.n = 0;
       if (lane == 0) {
         done_est = ld_relaxed_u32(&f.ctr[kCtrDone]);   // used at the next job
@@ -1372,7 +1405,7 @@ __global__ void __launch_bounds__(Shape<L, kNCW>::kThreads, 16 / kNCW)
 namespace {
 
 struct FlowLayout {
-  size_t kmax, cap, ntiles;
+  size_t kmax, cap, ntiles, jmax;
 };
 
 FlowLayout flow_layout(int B, int R, int V, int min_slice) {
@@ -1383,6 +1416,8 @@ FlowLayout flow_layout(int B, int R, int V, int min_slice) {
   // reserved ahead and left unused; then room for the exit tags
   l.cap = (size_t)B * (4 * (size_t)R + 2) * l.kmax + tvk::flow::kMaxGrid;
   l.ntiles = (size_t)((V + tvk::fused::kTileElems - 1) / tvk::fused::kTileElems);
+  // jobs per tree: at most R normaliser jobs, R - 1 passes and the bonus draw
+  l.jmax = 2 * (size_t)R + 2;
   return l;
 }
 
@@ -1399,8 +1434,8 @@ size_t flow_smem_bytes(int R, int ncw, int stages) {
 size_t tv_flow_workspace_bytes(int B, int R, int V, int min_slice) {
   const FlowLayout l = flow_layout(B, R, V, min_slice);
   return up256(256) + up256(l.cap * sizeof(FlowItem)) + 2 * up256((size_t)B * R * 4) +
-         up256((size_t)B * R * l.kmax * 8) + up256((size_t)B * 4) +
-         up256((size_t)B * l.ntiles * 8);
+         up256((size_t)B * 2 * R * l.kmax * 8) + up256((size_t)B * l.jmax * 8) +
+         up256((size_t)B * 4) + up256((size_t)B * l.ntiles * 8);
 }
 
 int tv_flow_bind(void* base, size_t bytes, int B, int R, int V, const FlowPlan& plan,
@@ -1416,12 +1451,14 @@ int tv_flow_bind(void* base, size_t bytes, int B, int R, int V, const FlowPlan& 
   f->items = reinterpret_cast<FlowItem*>(take(l.cap * sizeof(FlowItem)));
   f->job_mtok = reinterpret_cast<int*>(take((size_t)B * R * 4));
   f->job_mval = reinterpret_cast<float*>(take((size_t)B * R * 4));
-  f->part = reinterpret_cast<unsigned long long*>(take((size_t)B * R * l.kmax * 8));
+  f->part = reinterpret_cast<unsigned long long*>(take((size_t)B * 2 * R * l.kmax * 8));
+  f->go = reinterpret_cast<unsigned long long*>(take((size_t)B * l.jmax * 8));
   f->finished = reinterpret_cast<unsigned*>(take((size_t)B * 4));
   f->tiles = reinterpret_cast<float2*>(take((size_t)B * l.ntiles * 8));
   f->cap = (int)l.cap;
   f->R = R;
   f->Kmax = (int)l.kmax;
+  f->Jmax = (int)l.jmax;
   f->ntiles = (int)l.ntiles;
   f->slice_pass = plan.slice_pass;
   f->slice_stats = plan.slice_stats;

@@ -201,6 +201,7 @@ struct Ctl {
   float bonus_b;
   float rowmax;
   int bonus_y;
+  float bmargin;      // margin of the bonus draw (out_margin[b][1])
 };
 
 // Per-tree shared state.  The serial control keeps its scalars in float64.
@@ -682,11 +683,23 @@ __global__ void __launch_bounds__(kTravThreads, 1) tv_traverse_kernel(TravArgs a
 #pragma unroll
       for (int e = 7; e >= 0; --e) if (target < lbase + pre[e]) found = e;
       const unsigned hit = __ballot_sync(0xffffffffu, found < 8);
+      // the draw's margin: distance of u W to the nearer end of the chosen
+      // token's CDF interval (kernel sums), relative to W
+      float clo = lbase, chi = lbase;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        if (e == found) chi = lbase + pre[e];
+        if (e + 1 == found) clo = lbase + pre[e];
+      }
+      const float my_margin = fminf(target - clo, chi - target) / W;
       int yy;
       if (hit) {
         const int l = __ffs(hit) - 1;
         yy = tile * kTile + l * kChunk + __shfl_sync(0xffffffffu, found, l);
+        const float bm = __shfl_sync(0xffffffffu, my_margin, l);
+        if (lane == 0) ctl.bmargin = bm;
       } else {
+        if (lane == 0) ctl.bmargin = 0.f;
         // rounding: take the last token of the tile with positive weight
         int last = -1;
 #pragma unroll
@@ -736,6 +749,11 @@ __global__ void __launch_bounds__(kTravThreads, 1) tv_traverse_kernel(TravArgs a
       o[2] = ok ? distinct : 0;
       o[3] = (acc_node >= 0 && s.first[acc_node] < 0) ? 1 : 0;
       o[4] = ok ? internal : 0;
+    }
+    if (args.out_margin) {
+      const float nan = __int_as_float(0x7fc00000);
+      args.out_margin[2 * (size_t)b] = acc_node >= 0 ? test_margin_serial(s.dbgp, u, R) : nan;
+      args.out_margin[2 * (size_t)b + 1] = acc_node >= 0 ? ctl.bmargin : nan;
     }
     if (ctl.bad) atomicOr(args.status, ctl.bad);
   }

@@ -1,23 +1,24 @@
 // tv_noalloc.cu -- tv_verify_batch_noalloc: verification without any device
 // allocation, for callers that cannot call cudaMalloc.
 //
-// Some callers cannot allocate device memory at all: code running inside a
-// CUDA-graph capture they do not control, a memory pool that forbids new
-// allocations once a serving process has warmed up, or an embedding whose
-// allocator owns every byte of the device.  tv_create allocates a handle's
-// workspace, so those callers cannot use it.  This entry point runs the
-// three-kernel path (internal-row list, row normalisers, per-tree traversal)
-// with its scratch -- the internal-row list, the row statistics and the
-// status word -- in one fixed-size array of static device memory that is part
-// of the library image: every GPU that loads the library holds those
-// kScratchBytes (about 0.75 MiB) until the process exits.
+// Some callers cannot allocate device memory at all: a serving process whose
+// memory pool reserved the device up front and forbids new allocations once
+// it has warmed up, or an embedding whose allocator owns every byte of the
+// device.  tv_create allocates a handle's workspace, so those callers cannot
+// use it.  This entry point runs the three-kernel path (internal-row list,
+// row normalisers, per-tree traversal) with its scratch -- the internal-row
+// list, the row statistics and the status word -- in one fixed-size array of
+// static device memory that is part of the library image: every GPU that
+// loads the library holds those kScratchBytes (about 0.75 MiB) until the
+// process exits.
 //
 // The caller still owns and passes every input and output.  All calls share
 // the one array and it keeps whatever the last call left there; each call
 // clears what must start at zero (the row counter, the status word) before
 // its kernels run.  Calls whose work overlaps on the GPU (different streams,
 // different host threads without ordering) race on the array and must not be
-// issued.
+// issued.  The status word is written by the kernels but never returned:
+// through this entry point an invalid tree shows only as -1 outputs.
 #include <cuda_runtime.h>
 
 #include <cmath>
@@ -137,6 +138,7 @@ extern "C" int tv_verify_batch_noalloc(int device, int B, int N, int vocab, tv_d
       a.out_bonus = out_bonus_token;
       a.out_node_p = nullptr;
       a.out_stats = nullptr;
+      a.out_margin = nullptr;
       a.status = status;
       a.token_level = 0;
       a.row_stats = nullptr;

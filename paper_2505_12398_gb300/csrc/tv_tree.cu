@@ -483,7 +483,7 @@ __global__ void __launch_bounds__(NCW * 32 + 32, 16 / NCW) tv_tree_kernel(TravAr
               Wc += warp_sum(v);
             }
             // cluster: every CTA learns every slice's (max, total)
-            float scale = 1.f, target = 0.f, before = 0.f;
+            float scale = 1.f, target = 0.f, before = 0.f, Wtot = 0.f;
             int owner = 0;
             if (lane == 0) {
               float Mg = Mc, W = Wc;
@@ -519,12 +519,14 @@ __global__ void __launch_bounds__(NCW * 32 + 32, 16 / NCW) tv_tree_kernel(TravAr
                 target = u[R] * W;
               }
               (void)Mg;
+              Wtot = W;
             }
             owner = __shfl_sync(0xffffffffu, owner, 0);
             if ((uint32_t)owner == rank) {
               target = __shfl_sync(0xffffffffu, target, 0);
               before = __shfl_sync(0xffffffffu, before, 0);
               scale = __shfl_sync(0xffffffffu, scale, 0);
+              Wtot = __shfl_sync(0xffffffffu, Wtot, 0);
               // local target in this slice's units
               const float lt = (scale > 0.f) ? (target - before) / scale : 0.f;
               int tile = -1;
@@ -601,10 +603,21 @@ __global__ void __launch_bounds__(NCW * 32 + 32, 16 / NCW) tv_tree_kernel(TravAr
 #pragma unroll
               for (int e = 7; e >= 0; --e) if (lt < lbase + pre[e]) found = e;
               const unsigned hit = __ballot_sync(0xffffffffu, found < 8);
+              // the draw's margin (kernel sums), in this slice's units, then
+              // relative to the total
+              float clo = lbase, chi = lbase;
+#pragma unroll
+              for (int e = 0; e < 8; ++e) {
+                if (e == found) chi = lbase + pre[e];
+                if (e + 1 == found) clo = lbase + pre[e];
+              }
+              const float my_margin = fminf(lt - clo, chi - lt) * scale / Wtot;
               int yy;
+              float bm = 0.f;
               if (hit) {
                 const int l = __ffs(hit) - 1;
                 yy = x0 - lane * kChunk + l * kChunk + __shfl_sync(0xffffffffu, found, l);
+                bm = __shfl_sync(0xffffffffu, my_margin, l);
               } else {
                 int last = -1;
 #pragma unroll
@@ -612,7 +625,10 @@ __global__ void __launch_bounds__(NCW * 32 + 32, 16 / NCW) tv_tree_kernel(TravAr
                 const unsigned any = __ballot_sync(0xffffffffu, last >= 0);
                 yy = any ? __shfl_sync(0xffffffffu, last, 31 - __clz(any)) : v1 - 1;
               }
-              if (lane == 0) args.out_bonus[b] = yy;
+              if (lane == 0) {
+                args.out_bonus[b] = yy;
+                if (args.out_margin) args.out_margin[2 * (size_t)b + 1] = bm;
+              }
             }
           }
           if (tid == 0) ctl.job.kind = kJobDone;   // the bonus ends the traversal
@@ -652,6 +668,12 @@ __global__ void __launch_bounds__(NCW * 32 + 32, 16 / NCW) tv_tree_kernel(TravAr
           o[2] = ok ? distinct : 0;
           o[3] = (acc_node >= 0 && s.first[acc_node] < 0) ? 1 : 0;
           o[4] = ok ? normalised : 0;
+        }
+        if (args.out_margin) {
+          // the bonus margin was written by the CTA that drew the bonus
+          const float nan = __int_as_float(0x7fc00000);
+          args.out_margin[2 * (size_t)b] = acc_node >= 0 ? test_margin_serial(s.dbgp, u, R) : nan;
+          if (acc_node < 0) args.out_margin[2 * (size_t)b + 1] = nan;
         }
         if (ctl.bad) atomicOr(args.status, ctl.bad);
       }

@@ -8,15 +8,19 @@ for the bonus, relative to W) is at least ``TIE`` = 1e-5; trees with a
 near-tie are counted, compared up to the tie, and the GPU's choice at the tie
 is checked to be a valid one within the float32 error bound.
 
-Acceptance rates p of the tested nodes must agree within
-``P_RTOL`` * p + ``P_ATOL``.  S = sum_x [p M_b(x) - M_s(x)]_+ can cancel: its
-float32 value carries a relative error of about (element error) x kappa,
-kappa = sum over the positive part of p M_b / S, which the oracle records
-for every S (and the cancellation of each residual value a sibling's rate is
-later read from).  A rate that misses the 1e-5 bound but stays within
-``K_EPS`` * kappa * p (``K_EPS`` = 8 float32 ulps, the budget of the
-per-element exponential plus the summation) is counted as ill-conditioned
-and reported; anything beyond both bounds fails.
+Acceptance rates p of the tested nodes must agree within ``P_RTOL`` = 1e-5
+relative.  S = sum_x [p M_b(x) - M_s(x)]_+ can cancel: its float32 value
+carries a relative error of about (element error) x kappa, kappa = sum over
+the positive part of p M_b / S, which the oracle records for every S (and
+the cancellation of each residual value a sibling's rate is later read
+from).  A rate past the 1e-5 bar is an *escape*.  It is allowed only when
+its error is explained -- within ``K_EPS`` * kappa * p with kappa <=
+``KAPPA_MAX`` (``K_EPS`` = 8 float32 ulps, the budget of the per-element
+exponential plus the summation), or within the absolute floor ``P_ATOL`` --
+and in at most ``escape_budget(n)`` of a comparison's n trees (two, plus one
+per hundred).  Every escape is listed with its kappa and the
+S behind it; the reported maximum relative error covers every compared
+rate, escapes included.
 
 A rate below ``P_EQ0`` (far below float32's range and below any nonzero
 float32 uniform) is rejected with certainty exactly like a rate of 0, which
@@ -30,6 +34,7 @@ TIE = 1e-5
 P_RTOL = 1e-5
 P_ATOL = 1e-7
 K_EPS = 8 * 2.0 ** -24
+KAPPA_MAX = 1e4
 P_EQ0 = 1e-30
 
 
@@ -47,7 +52,8 @@ def to_numpy_inputs(inp, trees=None):
 def compare_tree(r, g_path, g_tau, g_bonus, g_p=None, g_stats=None):
     """Compare one tree; returns a dict of findings (raises nothing)."""
     out = {"exact": False, "tie": False, "ok": True, "why": [], "max_p_rel": 0.0,
-           "ill": 0, "max_kappa": 0.0}
+           "ill": 0, "floor": 0, "max_kappa": 0.0, "n_rates": 0, "escapes": [],
+           "test_tie": False}
     if "invalid" in r:
         ok = g_tau == -1 and g_bonus == -1 and (np.asarray(g_path) == -1).all()
         out.update(exact=ok, ok=ok)
@@ -63,15 +69,31 @@ def compare_tree(r, g_path, g_tau, g_bonus, g_p=None, g_stats=None):
     n_cmp = len(tests) if tie_at is None else tie_at + 1
     if g_p is not None:
         kap = r.get("kappa_at_test", [1.0] * len(tests))
-        for (node, u, p), k in zip(tests[:n_cmp], kap):
+        Ss = r.get("S_at_test", [float("nan")] * len(tests))
+        for (node, u, p), k, S in zip(tests[:n_cmp], kap, Ss):
             gp = float(g_p[node])
             err = abs(gp - p)
-            if err <= P_RTOL * p + P_ATOL:
-                if p > 0:
-                    out["max_p_rel"] = max(out["max_p_rel"], err / p)
-            elif err <= K_EPS * k * p:
+            if p < P_EQ0:
+                # a rate below float32's range: rejected with certainty either way
+                if not gp < P_EQ0:
+                    out["ok"] = False
+                    out["why"].append(f"p of node {node}: gpu {gp!r} oracle {p!r}")
+                continue
+            out["n_rates"] += 1
+            out["max_p_rel"] = max(out["max_p_rel"], err / p)
+            if err <= P_RTOL * p:
+                continue
+            # beyond 1e-5 relative: an escape, allowed only within the bound
+            # that explains it (float32 cancellation in S, or the absolute floor)
+            esc = {"node": node, "gpu": gp, "oracle": p, "kappa": k, "S": S,
+                   "rel": err / p if p > 0 else float("inf")}
+            if err <= K_EPS * k * p and k <= KAPPA_MAX:
                 out["ill"] += 1
                 out["max_kappa"] = max(out["max_kappa"], k)
+                out["escapes"].append(esc)
+            elif err <= P_ATOL:
+                out["floor"] += 1
+                out["escapes"].append(esc)
             else:
                 out["ok"] = False
                 out["why"].append(f"p of node {node}: gpu {gp!r} oracle {p!r} (kappa {k:.3g})")
@@ -81,6 +103,7 @@ def compare_tree(r, g_path, g_tau, g_bonus, g_p=None, g_stats=None):
                 out["why"].append(f"pruned node {c} has gpu p {g_p[c]}")
     if tie_at is not None:
         out["tie"] = True
+        out["test_tie"] = True
         return out
     path = list(np.asarray(g_path)[: max(g_tau, 0)])
     if g_tau != r["tau"] or path != r["path"]:
@@ -118,9 +141,12 @@ def compare_tree(r, g_path, g_tau, g_bonus, g_p=None, g_stats=None):
 
 
 def compare_batch(details, g_path, g_tau, g_bonus, g_p=None, g_stats=None):
-    """details: {tree index: oracle result}.  Returns summary dict."""
-    summ = {"trees": 0, "exact": 0, "ties": 0, "bad": [], "max_p_rel": 0.0, "ill": 0,
-            "max_kappa": 0.0}
+    """details: {tree index: oracle result}.  Returns summary dict: counts,
+    the true maximum relative error over every compared rate (those that
+    escaped the 1e-5 bar included) and the list of escapes (tree, node, GPU
+    and oracle rate, kappa and the S behind it)."""
+    summ = {"trees": 0, "exact": 0, "ties": 0, "test_ties": 0, "bad": [], "max_p_rel": 0.0,
+            "ill": 0, "floor": 0, "max_kappa": 0.0, "n_rates": 0, "escapes": []}
     for b, r in details.items():
         c = compare_tree(r, g_path[b], int(g_tau[b]), int(g_bonus[b]),
                          None if g_p is None else g_p[b],
@@ -128,9 +154,33 @@ def compare_batch(details, g_path, g_tau, g_bonus, g_p=None, g_stats=None):
         summ["trees"] += 1
         summ["exact"] += int(c["exact"])
         summ["ties"] += int(c["tie"])
+        summ["test_ties"] += int(c["test_tie"])
         summ["max_p_rel"] = max(summ["max_p_rel"], c["max_p_rel"])
         summ["ill"] += c["ill"]
+        summ["floor"] += c["floor"]
+        summ["n_rates"] += c["n_rates"]
+        summ["escapes"] += [dict(e, tree=b) for e in c["escapes"]]
         summ["max_kappa"] = max(summ["max_kappa"], c["max_kappa"])
         if not c["ok"]:
             summ["bad"].append((b, c["why"]))
     return summ
+
+
+def escape_budget(n_trees):
+    """Trees allowed to hold rates past the 1e-5 relative bar in one
+    comparison: two, plus one per hundred trees.  Escapes cluster by tree
+    (an ill-conditioned S feeds every rate below it), so they are budgeted per
+    tree.  Measured on every GPU parity case: 44 of 11181 rates (0.39 %) in 27
+    of 3766 trees (0.7 %), at most two trees per comparison, every one
+    explained by the float32 cancellation bound or the absolute floor."""
+    return 2 + n_trees // 100
+
+
+def escaped_trees(summ):
+    return len({e["tree"] for e in summ["escapes"]})
+
+
+def assert_rate_budget(summ):
+    """Every escape past the 1e-5 bar was explained (compare_tree), and there
+    are no more of them than the budget allows."""
+    assert escaped_trees(summ) <= escape_budget(summ["trees"]), summ["escapes"]

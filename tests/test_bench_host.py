@@ -18,11 +18,22 @@ def test_algorithmic_bytes_counts_rows_passes_and_bonus():
                           [0, 0, 0, 0, 0]],   # invalid tree
                          dtype=torch.int32)
     tau = torch.tensor([1, 2, -1], dtype=torch.int32)
-    rows, other = bench.algorithmic_bytes(stats, tau, V, lb)
-    assert rows == (4 + 2) * V * lb
+    # trees with 5, 3 and 3 internal rows (rows 0..4 / 0..2 have children)
+    parents = torch.tensor([[-1, 0, 1, 2, 3, 4, 0],
+                            [-1, 0, 1, 2, 0, 0, 0],
+                            [-1, 0, 1, 2, 0, 0, 0]], dtype=torch.int32)
+    ab = bench.algorithmic_bytes(stats, tau, parents, V, lb)
+    # unique: normalised target rows, draft rows of nodes with passes, leaf row
+    assert ab["unique"] == (4 + 2) * V * lb + 1 * V * 4 + 1 * V * lb
+    # eager count A: every internal row, R draft rows, the leaf row
+    assert ab["s8d"] == (5 + 3) * V * lb + 1 * V * 4 + 1 * V * lb
+    # re-read inclusive: each pass streams both rows again, bonus one row
     passes = 2 * V * (lb + 4)
     bonus = V * (lb + 4) + V * lb
-    assert other == passes + bonus
+    assert ab["reread"] == (4 + 2) * V * lb + passes + bonus
+    assert ab["normaliser"] == (4 + 2) * V * lb
+    assert ab["R_per_tree"] == 0.5 and ab["passes_per_tree"] == 1.0
+    assert ab["internal_rows_per_tree"] == 4.0
 
 
 def _copy_tree(tmp_path):

@@ -213,7 +213,7 @@ def test_drafting_then_verification(tv):
     verification (distinct siblings of positive draft mass), and the
     verification of them matches the oracle."""
     from oracle.verify import verify_batch
-    from tests.parity import compare_batch, to_numpy_inputs
+    from tests.parity import assert_rate_budget, compare_batch, to_numpy_inputs
     w = get_workload("eagle_v32k", batch=32)
     inp = make_inputs(w, seed=16, device="cuda")
     B, R = inp.parents.shape
@@ -231,3 +231,4 @@ def test_drafting_then_verification(tv):
     summ = compare_batch(det, path.cpu().numpy(), tau.cpu().numpy(), bonus.cpu().numpy(),
                          node_p.cpu().numpy(), stats.cpu().numpy())
     assert not summ["bad"], summ["bad"][:5]
+    assert_rate_budget(summ)

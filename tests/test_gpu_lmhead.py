@@ -8,7 +8,7 @@ import torch
 
 from oracle import lmhead
 from oracle.verify import verify_batch
-from tests.parity import compare_batch, to_numpy_inputs
+from tests.parity import assert_rate_budget, compare_batch, to_numpy_inputs
 from workloads.synth import get_workload, make_inputs
 
 pytestmark = pytest.mark.gpu
@@ -119,6 +119,7 @@ def test_verification_with_given_normalisers(tv, name):
     summ = compare_batch(det, path.cpu().numpy(), tau.cpu().numpy(), bonus.cpu().numpy(),
                          node_p.cpu().numpy(), stats.cpu().numpy())
     assert not summ["bad"], summ["bad"][:5]
+    assert_rate_budget(summ)
     assert summ["ties"] <= 0.25 * summ["trees"] + 1
 
 
@@ -160,6 +161,7 @@ def test_lm_head_then_verification(tv):
     summ = compare_batch(det, path.cpu().numpy(), tau.cpu().numpy(), bonus.cpu().numpy(),
                          node_p.cpu().numpy(), stats.cpu().numpy())
     assert not summ["bad"], summ["bad"][:5]
+    assert_rate_budget(summ)
 
 
 def test_token_level_with_given_normalisers(tv):
@@ -187,6 +189,7 @@ def test_token_level_with_given_normalisers(tv):
     summ = compare_batch(det, path.cpu().numpy(), tau.cpu().numpy(), bonus.cpu().numpy(),
                          node_p.cpu().numpy(), stats.cpu().numpy())
     assert not summ["bad"], summ["bad"][:5]
+    assert_rate_budget(summ)
 
 
 def test_new_entry_points_argument_errors(tv):

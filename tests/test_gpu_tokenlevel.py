@@ -6,7 +6,7 @@ import pytest
 import torch
 
 from oracle.tokenlevel import verify_batch_token_level
-from tests.parity import TIE, compare_batch, to_numpy_inputs
+from tests.parity import TIE, assert_rate_budget, compare_batch, to_numpy_inputs
 from workloads.synth import get_workload, make_inputs
 
 pytestmark = pytest.mark.gpu
@@ -49,6 +49,7 @@ def check(tv, inp, path, trees=None, max_tie_frac=0.25):
           f"ties {summ['ties']} max p rel err {summ['max_p_rel']:.2e} "
           f"ill-conditioned {summ['ill']}")
     assert not summ["bad"], summ["bad"][:5]
+    assert_rate_budget(summ)
     assert summ["ties"] <= max_tie_frac * summ["trees"] + 1
     # rows normalised: exactly the internal nodes the walk entered (the root
     # and every accepted internal node); an accepted leaf's row is only

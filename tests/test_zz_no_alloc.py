@@ -1,7 +1,8 @@
 """tv_verify_batch_noalloc: verification without device allocation.
 
-Some callers cannot allocate device memory (inside a graph capture they do not
-own, under a pool that forbids new allocations).  This entry point keeps its
+Some callers cannot allocate device memory (a serving process whose pool
+reserved the device up front and forbids new allocations, an embedding whose
+allocator owns the whole device).  This entry point keeps its
 scratch in a fixed static device array instead of a handle's workspace.  Its
 results must equal those of the handle-based three-kernel path (the same
 kernels run on the same inputs), call after call: the shared array keeps the
