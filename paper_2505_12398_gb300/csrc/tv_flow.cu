@@ -73,8 +73,7 @@ constexpr int kItemNop = 6;         // FlowItem::kind of a reserved slot that ca
 struct ItemSlot {
   int b, node, row, slice;
   int kind, slice_len, nmask, pad0;
-  float alpha1, beta, rowmax;
-  int par;                 // parity of the job's sequence number (its partials buffer)
+  float alpha1, beta, rowmax, pad1;
 };
 
 struct StageMeta {
@@ -90,16 +89,7 @@ struct Shared {
   Job fjob;                          // a job posted from `ahead`
   float2 pbuf[kPBuf];                // the own job's partials, as read by the poll
   int jkind, jrows, jK, jslice, outstanding;
-  int jseq;                          // sequence number of the own tree's current job
 };
-
-// Partial of (tree b, job parity par, row r of the job, slice k).  Jobs
-// alternate between two buffers, so a job's slices may be reset and written
-// while the previous job's partials are still being read.
-__device__ __forceinline__ unsigned long long* part_at(const FlowArgs& f, int b, int par, int r,
-                                                       int k) {
-  return f.part + (((size_t)b * 2 + par) * f.R + r) * f.Kmax + k;
-}
 
 __device__ __forceinline__ unsigned ld_relaxed_u32(const unsigned* p) {
   unsigned v;
@@ -257,7 +247,6 @@ __device__ void fetcher_role(const TravArgs& a, const FlowArgs& f, const Smem& m
         it.kind = w[1].x; it.slice_len = w[1].y; it.nmask = w[1].z;
         it.alpha1 = __int_as_float(w[2].x); it.beta = __int_as_float(w[2].y);
         it.rowmax = __int_as_float(w[2].z);
-        it.par = w[2].w;
         int* mt = m.mtok + slot * R;
         float* mv = m.mval + slot * R;
         const int ni = min(w[1].z, kFlowInlineMask);
@@ -364,7 +353,7 @@ __device__ void consumer_role(const TravArgs& a, const FlowArgs& f, const Smem& 
   int stage = 0, phase = 0;
   unsigned red_phase = 0u;   // parity bit per stage of red_bar (warp 0 waits on it)
   // the slice in progress
-  int kind = 0, b = 0, row_idx = 0, slice = 0, nmask = 0, slot = 0, x0 = 0, x1 = 0, par = 0;
+  int kind = 0, b = 0, row_idx = 0, slice = 0, nmask = 0, slot = 0, x0 = 0, x1 = 0;
   float alpha1 = 0.f, beta = 0.f, rowmax = 0.f;
   float m_run = TV_NEG_INF;
   Comp acc;
@@ -379,7 +368,6 @@ __device__ void consumer_role(const TravArgs& a, const FlowArgs& f, const Smem& 
     if (meta.flags & kStageFirst) {
       const ItemSlot& it = m.sh->slots[meta.slot];
       kind = it.kind; b = it.b; row_idx = it.row; slice = it.slice; nmask = it.nmask;
-      par = it.par;
       alpha1 = it.alpha1; beta = it.beta; rowmax = it.rowmax;
       slot = meta.slot;
       x0 = slice * it.slice_len;
@@ -619,7 +607,7 @@ __device__ void consumer_role(const TravArgs& a, const FlowArgs& f, const Smem& 
           fence_gpu();   // the tiles before the partial that announces them
         }
         if (lane == 0) {
-          st_relaxed_u64(part_at(f, b, par, row_idx, slice), pack_part(px, py));
+          st_relaxed_u64(f.part + ((size_t)b * R + row_idx) * f.Kmax + slice, pack_part(px, py));
           mbar_arrive(&m.empty_bar[stage]);   // only now may the stage (and red[stage]) be reused
         }
       } else if (lane == 0) {
@@ -694,8 +682,7 @@ __device__ __forceinline__ void reserve_next(const FlowArgs& f, int V, int B, in
 // use the slots reserved in `spec`; otherwise those become "no work" items.
 __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const FlowArgs& f,
                          int b, int V, int lane, unsigned done, Reserve spec, const Job& j,
-                         const int* mask_tok, const float* mask_val, int seq) {
-  const int par = seq & 1;
+                         const int* mask_tok, const float* mask_val) {
   const bool stats = (j.kind == kJobStats);
   const int n_rows = stats ? j.n_rows : 1;
   const bool use_spec = spec.n > 0 && j.kind == kJobPass;
@@ -711,7 +698,7 @@ __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const
   // the job's partial slots start as "not yet"
   for (int q = lane; q < n; q += 32) {
     const int r = q / K;
-    __stcg(part_at(f, b, par, r, q - r * K), kNoPart);
+    __stcg(f.part + ((size_t)b * R + r) * f.Kmax + (q - r * K), kNoPart);
   }
   unsigned base = spec.base;
   if (!use_spec) {
@@ -728,7 +715,7 @@ __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const
   if (spec.n > 0 && !use_spec) nop_bodies(f, spec.base, spec.n, lane);
   const int4 w1 = make_int4(j.kind, slice, nmask, 0);
   const int4 w2 = make_int4(__float_as_int(j.alpha1), __float_as_int(j.beta),
-                            __float_as_int(j.rowmax), par);
+                            __float_as_int(j.rowmax), 0);
   int tk[kFlowInlineMask];
   float vk[kFlowInlineMask];
 #pragma unroll
@@ -769,7 +756,6 @@ __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const
     sh.jrows = n_rows;
     sh.jK = K;
     sh.jslice = slice;
-    sh.jseq = seq;
   }
 }
 
@@ -782,7 +768,6 @@ __device__ void owner_new_tree(const TravArgs& a, const TreeSmem& s, Shared& sh,
   const typename L::elem* logits = reinterpret_cast<const typename L::elem*>(a.logits);
   if (lane == 0) {
     sh.outstanding = 0;
-    sh.jseq = -1;
     sh.ahead.ok = 0;
     Ctl& c = sh.ctl;
     c.bad = 0u;
@@ -891,7 +876,7 @@ __device__ void owner_combine(const TravArgs& a, const FlowArgs& f, const TreeSm
   const bool in_smem = sh.outstanding <= kPBuf;
   auto part_of = [&](int r, int k) -> float2 {
     return in_smem ? sh.pbuf[r * K + k]
-                   : unpack_part(__ldcg(part_at(f, b, sh.jseq & 1, r, k)));
+                   : unpack_part(__ldcg(f.part + (row0 + r) * f.Kmax + k));
   };
   if (sh.jkind == kJobStats) {
     // the rows' normalisers from their slices, one lane per row ...
@@ -1188,7 +1173,7 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
       for (int q = lane; q < nout; q += 32) {
         const int r = q / K;
         const unsigned long long v =
-            ld_relaxed_u64(part_at(f, my_tree, sh.jseq & 1, r, q - r * K));
+            ld_relaxed_u64(f.part + ((size_t)my_tree * R + r) * f.Kmax + (q - r * K));
         if (v == kNoPart) all = false;
         else if (q < kPBuf) sh.pbuf[q] = unpack_part(v);
       }
@@ -1269,13 +1254,13 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
           __syncwarp();
           if (post_first) {
             post_job(s, sh, a, f, my_tree, V, lane, __shfl_sync(0xffffffffu, done_est, 0),
-                     spec, sh.fjob, m.mtok2, s.mask_val, sh.jseq + 1);
+                     spec, sh.fjob, m.mtok2, s.mask_val);
             if (lane == 0) control_step_ahead(s, sh.ctl, sh.ahead, accept != 0);
           } else {
             if (lane == 0) control_step_ahead(s, sh.ctl, sh.ahead, accept != 0);
             __syncwarp();
             post_job(s, sh, a, f, my_tree, V, lane, __shfl_sync(0xffffffffu, done_est, 0),
-                     spec, sh.ctl.job, s.mask_tok, s.mask_val, sh.jseq + 1);
+                     spec, sh.ctl.job, s.mask_tok, s.mask_val);
           }
           spec.n = 0;
           if (lane == 0) {
@@ -1312,7 +1297,7 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
       }
     } else {
       post_job(s, sh, a, f, my_tree, V, lane, __shfl_sync(0xffffffffu, done_est, 0), spec,
-               sh.ctl.job, s.mask_tok, s.mask_val, sh.jseq + 1);
+               sh.ctl.job, s.mask_tok, s.mask_val);
       spec.n = 0;
       if (lane == 0) {
         done_est = ld_relaxed_u32(&f.ctr[kCtrDone]);   // used at the next job
@@ -1405,7 +1390,7 @@ __global__ void __launch_bounds__(Shape<L, kNCW>::kThreads, 16 / kNCW)
 namespace {
 
 struct FlowLayout {
-  size_t kmax, cap, ntiles, jmax;
+  size_t kmax, cap, ntiles;
 };
 
 FlowLayout flow_layout(int B, int R, int V, int min_slice) {
@@ -1416,8 +1401,6 @@ FlowLayout flow_layout(int B, int R, int V, int min_slice) {
   // reserved ahead and left unused; then room for the exit tags
   l.cap = (size_t)B * (4 * (size_t)R + 2) * l.kmax + tvk::flow::kMaxGrid;
   l.ntiles = (size_t)((V + tvk::fused::kTileElems - 1) / tvk::fused::kTileElems);
-  // jobs per tree: at most R normaliser jobs, R - 1 passes and the bonus draw
-  l.jmax = 2 * (size_t)R + 2;
   return l;
 }
 
@@ -1434,8 +1417,8 @@ size_t flow_smem_bytes(int R, int ncw, int stages) {
 size_t tv_flow_workspace_bytes(int B, int R, int V, int min_slice) {
   const FlowLayout l = flow_layout(B, R, V, min_slice);
   return up256(256) + up256(l.cap * sizeof(FlowItem)) + 2 * up256((size_t)B * R * 4) +
-         up256((size_t)B * 2 * R * l.kmax * 8) + up256((size_t)B * l.jmax * 8) +
-         up256((size_t)B * 4) + up256((size_t)B * l.ntiles * 8);
+         up256((size_t)B * R * l.kmax * 8) + up256((size_t)B * 4) +
+         up256((size_t)B * l.ntiles * 8);
 }
 
 int tv_flow_bind(void* base, size_t bytes, int B, int R, int V, const FlowPlan& plan,
@@ -1451,14 +1434,12 @@ int tv_flow_bind(void* base, size_t bytes, int B, int R, int V, const FlowPlan& 
   f->items = reinterpret_cast<FlowItem*>(take(l.cap * sizeof(FlowItem)));
   f->job_mtok = reinterpret_cast<int*>(take((size_t)B * R * 4));
   f->job_mval = reinterpret_cast<float*>(take((size_t)B * R * 4));
-  f->part = reinterpret_cast<unsigned long long*>(take((size_t)B * 2 * R * l.kmax * 8));
-  f->go = reinterpret_cast<unsigned long long*>(take((size_t)B * l.jmax * 8));
+  f->part = reinterpret_cast<unsigned long long*>(take((size_t)B * R * l.kmax * 8));
   f->finished = reinterpret_cast<unsigned*>(take((size_t)B * 4));
   f->tiles = reinterpret_cast<float2*>(take((size_t)B * l.ntiles * 8));
   f->cap = (int)l.cap;
   f->R = R;
   f->Kmax = (int)l.kmax;
-  f->Jmax = (int)l.jmax;
   f->ntiles = (int)l.ntiles;
   f->slice_pass = plan.slice_pass;
   f->slice_stats = plan.slice_stats;

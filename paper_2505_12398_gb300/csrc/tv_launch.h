@@ -77,13 +77,12 @@ struct FlowArgs {
   FlowItem* items;               // [cap] queue slots
   int* job_mtok;                 // [B][R] removed tokens of a tree's current job row
   float* job_mval;               // [B][R] their stored masses (bonus residual)
-  unsigned long long* part;      // [B][2][R][Kmax] partial (x, y) per (job parity, row,
-                                 // slice); all ones until the slice is done
-  unsigned long long* go;        // [B][Jmax] release word of each job posted ahead
+  unsigned long long* part;      // [B][R][Kmax] partial (x, y) per (row, slice); all ones
+                                 // until the slice is done
   unsigned* finished;            // [B] epoch of the call that finished the tree
   float2* tiles;                 // [B][ntiles] per-tile sums of the bonus draw
   unsigned long long epoch;      // differs between calls sharing the workspace
-  int cap, R, Kmax, ntiles, Jmax;
+  int cap, R, Kmax, ntiles;
   int slice_pass, slice_stats;   // largest tokens per slice (multiples of 256)
   int slice_min;                 // smallest tokens per slice (multiple of 256)
   int withhold_tree;             // test hook: this tree's jobs are never published (-1: none)
