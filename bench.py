@@ -441,19 +441,11 @@ def main():
         torch.cuda.synchronize(dev)
         e_ms = x0.elapsed_time(x1)
         e_ms_max = max_over_ranks(e_ms, world, dev)
-        # what the host entry point copied; with pinned inputs it reads the
-        # rows it needs in place, so the bytes that cross the host link are
-        # the copies plus those reads, at most the re-read-inclusive row bytes
-        # (L2 hits only lower it)
+        # what the host entry point copied (it skips the draft rows of leaves)
         h2d, d2h = v.last_host_copy_bytes()
-        in_place = v.last_host_read_in_place()
         assert torch.equal(hout[1], out[1].cpu()), "host entry point disagrees"
-        row_reads = ab["reread"] if in_place else 0
         e2e = {"value": round(whole_job_rate(B, world, ks, e_ms_max), 3), "unit": "trees/s",
-               "h2d_bytes_per_step": int(h2d) + int(row_reads),
-               "d2h_bytes_per_step": int(d2h), "steps": ks,
-               "rows_read_in_place": bool(in_place), "h2d_copied_bytes": int(h2d),
-               "h2d_row_reads_upper_bound": int(row_reads)}
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": ks}
 
     # CPU baseline: the oracle on host cores, bounded sample of the same batch
     cpu = None

@@ -204,22 +204,14 @@ int tv_verify_batch_debug(tv_handle* h, int B, int N, const int32_t* parents,
                           void* cuda_stream);
 
 /*
- * tv_verify_batch_host -- the same verification from HOST buffers: runs
- * tv_verify_batch on cuda_stream, copies the three outputs back and
- * synchronises the stream before returning.  All pointers are host pointers
- * with the layouts above.  The verification reads only a fraction of the
- * rows (the lazily normalised chains, the rows of nodes with a rejection, one
- * bonus row), so how the rows reach the GPU matters:
- *   - target_logits and draft_probs both in pinned (page-locked) host memory
- *     that the device can address (cudaHostAlloc or registered memory on a
- *     system with unified addressing; NVLink-C2C on Grace): the kernels read
- *     the rows they need in place, and only the tree arrays and uniforms are
- *     copied (into a small handle-owned buffer);
- *   - otherwise: everything is copied to device staging owned by the handle
- *     (allocated on first use, sized by tv_create's limits), except the draft
- *     rows of nodes without children, which are never read (one 2-D copy per
- *     run of rows with children when all trees share their parents).
- * Errors as tv_verify_batch.
+ * tv_verify_batch_host -- the same verification from HOST buffers: copies the
+ * inputs to device staging owned by the handle (allocated on first use, sized
+ * by tv_create's limits), runs tv_verify_batch on cuda_stream, copies the
+ * three outputs back and synchronises the stream before returning.  All
+ * pointers are host pointers with the layouts above; pinned (page-locked)
+ * memory gives the fastest copies.  Draft rows of nodes without children are
+ * never read and are not copied (one 2-D copy per run of rows with children
+ * when all trees share their parents).  Errors as tv_verify_batch.
  */
 int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
                          const int32_t* draft_tokens, const void* target_logits,
@@ -230,20 +222,10 @@ int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
 
 /*
  * tv_last_host_copy_bytes -- bytes the last successful tv_verify_batch_host
- * call on this handle copied host to device (*h2d) and device to host (*d2h)
- * with copy operations (rows read in place are not counted).
+ * call on this handle copied host to device (*h2d) and device to host (*d2h).
  * Either pointer may be NULL.  Errors: TV_ERR_INVALID_ARG (no handle).
  */
 int tv_last_host_copy_bytes(tv_handle* h, uint64_t* h2d, uint64_t* d2h);
-
-/*
- * tv_last_host_read_in_place -- *in_place = 1 if the last successful
- * tv_verify_batch_host call on this handle read the rows in place from host
- * memory (tv_last_host_copy_bytes then counts only the copied tree arrays,
- * uniforms and outputs), 0 if it staged them.
- * Errors: TV_ERR_INVALID_ARG (no handle or null pointer).
- */
-int tv_last_host_read_in_place(tv_handle* h, int* in_place);
 
 /*
  * tv_lm_head -- the target model's last layer fused with the row normalisers

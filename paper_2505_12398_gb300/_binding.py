@@ -54,7 +54,6 @@ _SIGS = {
     "tv_lm_head": (_I, [_P, _I, _I, _P, _P, _F, _P, _P, _P]),
     "tv_draft_children": (_I, [_P, _I, _I, _P, _P, _P, _P, _P]),
     "tv_last_host_copy_bytes": (_I, [_P, _P, _P]),
-    "tv_last_host_read_in_place": (_I, [_P, _P]),
     "tv_get_status": (_I, [_P, ctypes.POINTER(ctypes.c_uint32)]),
     "tv_debug_withhold_job": (_I, [_P, _I]),
     "tv_destroy": (_I, [_P]),
@@ -285,10 +284,9 @@ class Verifier:
 
     def verify_host(self, parents, tokens, logits, drafts, temperature, uniforms,
                     out, stream=None):
-        """Same verification from host (CPU) tensors, outputs into ``out`` =
-        (path, tau, bonus) host tensors; synchronises.  Pinned logits and draft
-        rows are read in place by the kernels, others are copied first
-        (tv_verify_batch_host)."""
+        """Same verification from host (CPU, ideally pinned) tensors; copies in,
+        verifies, copies the outputs into ``out`` = (path, tau, bonus) host
+        tensors and synchronises."""
         B, R = parents.shape
         N = R - 1
         path, tau, bonus = out
@@ -308,15 +306,6 @@ class Verifier:
         if rc != 0:
             raise LibraryError("tv_last_host_copy_bytes", rc, self.lib)
         return h2d.value, d2h.value
-
-    def last_host_read_in_place(self):
-        """True if the last verify_host call read the rows in place from pinned
-        host memory instead of copying them (tv_last_host_read_in_place)."""
-        on = ctypes.c_int()
-        rc = self.lib.tv_last_host_read_in_place(self.handle, ctypes.byref(on))
-        if rc != 0:
-            raise LibraryError("tv_last_host_read_in_place", rc, self.lib)
-        return bool(on.value)
 
     def set_phase_timing(self, enable=True):
         rc = self.lib.tv_set_phase_timing(self.handle, 1 if enable else 0)

@@ -46,10 +46,7 @@ struct tv_handle {
   // its last call copied each way
   char* stage = nullptr;
   size_t stage_bytes = 0;
-  char* small_stage = nullptr;   // tree arrays and outputs only (rows read in place)
-  size_t small_stage_bytes = 0;
   uint64_t host_h2d_bytes = 0, host_d2h_bytes = 0;
-  int host_in_place = 0;         // the last host call read the rows in place
   // optional per-kernel timing events
   bool timing = false;
   bool timed_call = false;
@@ -384,82 +381,6 @@ int tv_verify_batch_debug(tv_handle* h, int B, int N, const int32_t* parents,
                      out_stats, cuda_stream, nullptr, out_margin);
 }
 
-namespace {
-
-// The device address of pinned, mapped host memory (nullptr for anything else:
-// device memory, pageable memory, unknown pointers).
-const void* device_view_of_host(const void* p) {
-  cudaPointerAttributes at;
-  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
-    cudaGetLastError();
-    return nullptr;
-  }
-  if (at.type != cudaMemoryTypeHost || at.devicePointer == nullptr) return nullptr;
-  return at.devicePointer;
-}
-
-// tv_verify_batch_host with the rows read in place: only the tree arrays and
-// uniforms are copied (into a small handle-owned buffer), the kernels stream
-// the logit and draft rows they need straight from host memory.
-int verify_host_in_place(tv_handle* h, int B, int N, const int32_t* parents,
-                         const int32_t* tokens, const void* d_logit, const float* d_draft,
-                         float temperature, const float* uniforms, int32_t* out_path,
-                         int32_t* out_len, int32_t* out_bonus, cudaStream_t st) {
-  const size_t R = static_cast<size_t>(N) + 1;
-  const size_t n_tree = static_cast<size_t>(B) * R * sizeof(int32_t);
-  const size_t n_unif = static_cast<size_t>(B) * (R + 1) * sizeof(float);
-  const size_t n_path = static_cast<size_t>(B) * N * sizeof(int32_t);
-  const size_t n_out = static_cast<size_t>(B) * sizeof(int32_t);
-  auto up = [](size_t x) { return (x + 255) & ~static_cast<size_t>(255); };
-  const size_t need = 2 * up(n_tree) + up(n_unif) + up(n_path) + 2 * up(n_out);
-  if (need > h->small_stage_bytes) {
-    const size_t Rm = static_cast<size_t>(h->max_nodes) + 1;
-    const size_t Bm = static_cast<size_t>(h->max_batch);
-    const size_t cap = 2 * up(Bm * Rm * 4) + up(Bm * (Rm + 1) * 4) + up(Bm * (Rm - 1) * 4) +
-                       2 * up(Bm * 4);
-    if (h->small_stage) cudaFree(h->small_stage);
-    h->small_stage = nullptr;
-    h->small_stage_bytes = 0;
-    if (cudaMalloc(&h->small_stage, cap) != cudaSuccess) {
-      cudaGetLastError();
-      return TV_ERR_CUDA;
-    }
-    h->small_stage_bytes = cap;
-  }
-  char* p = h->small_stage;
-  int32_t* d_par = reinterpret_cast<int32_t*>(p); p += up(n_tree);
-  int32_t* d_tok = reinterpret_cast<int32_t*>(p); p += up(n_tree);
-  float* d_unif = reinterpret_cast<float*>(p); p += up(n_unif);
-  int32_t* d_path = reinterpret_cast<int32_t*>(p); p += up(n_path);
-  int32_t* d_len = reinterpret_cast<int32_t*>(p); p += up(n_out);
-  int32_t* d_bonus = reinterpret_cast<int32_t*>(p);
-  bool ok = cudaMemcpyAsync(d_par, parents, n_tree, cudaMemcpyHostToDevice, st) == cudaSuccess &&
-            cudaMemcpyAsync(d_tok, tokens, n_tree, cudaMemcpyHostToDevice, st) == cudaSuccess &&
-            cudaMemcpyAsync(d_unif, uniforms, n_unif, cudaMemcpyHostToDevice, st) == cudaSuccess;
-  if (!ok) {
-    cudaGetLastError();
-    return TV_ERR_CUDA;
-  }
-  int rc = verify_impl(h, B, N, d_par, d_tok, d_logit, d_draft, temperature, d_unif, d_path,
-                       d_len, d_bonus, nullptr, nullptr, st);
-  if (rc != TV_OK) return rc;
-  ok = (N == 0 || cudaMemcpyAsync(out_path, d_path, n_path, cudaMemcpyDeviceToHost, st) ==
-                      cudaSuccess) &&
-       cudaMemcpyAsync(out_len, d_len, n_out, cudaMemcpyDeviceToHost, st) == cudaSuccess &&
-       cudaMemcpyAsync(out_bonus, d_bonus, n_out, cudaMemcpyDeviceToHost, st) == cudaSuccess &&
-       cudaStreamSynchronize(st) == cudaSuccess;
-  if (!ok) {
-    cudaGetLastError();
-    return TV_ERR_CUDA;
-  }
-  h->host_h2d_bytes = 2 * n_tree + n_unif;
-  h->host_d2h_bytes = (N > 0 ? n_path : 0) + 2 * n_out;
-  h->host_in_place = 1;
-  return TV_OK;
-}
-
-}  // namespace
-
 int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
                          const int32_t* draft_tokens, const void* target_logits,
                          const float* draft_probs, float temperature,
@@ -475,15 +396,6 @@ int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
   const size_t R = static_cast<size_t>(N) + 1;
   const size_t V = static_cast<size_t>(h->vocab);
-  // Logits and draft rows in pinned host memory that the device can address
-  // (on a Grace system over NVLink-C2C) are read in place by the kernels:
-  // the traversal reads only the rows it needs, a fraction of the batch.
-  const void* z_logit = device_view_of_host(target_logits);
-  const void* z_draft = device_view_of_host(draft_probs);
-  if (z_logit && z_draft)
-    return verify_host_in_place(h, B, N, parents, draft_tokens, z_logit,
-                                static_cast<const float*>(z_draft), temperature, uniforms,
-                                out_accepted_path, out_accept_len, out_bonus_token, st);
   const size_t n_tree = static_cast<size_t>(B) * R * sizeof(int32_t);
   const size_t n_logit = static_cast<size_t>(B) * R * V * logit_bytes(h);
   const size_t n_draft = static_cast<size_t>(B) * R * V * sizeof(float);
@@ -541,7 +453,6 @@ int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
     return TV_ERR_CUDA;
   }
   h->host_h2d_bytes = 2 * n_tree + n_unif + n_logit + draft_bytes;
-  h->host_in_place = 0;
   h->host_d2h_bytes = (N > 0 ? n_path : 0) + 2 * n_out;
   return TV_OK;
 }
@@ -550,12 +461,6 @@ int tv_last_host_copy_bytes(tv_handle* h, uint64_t* h2d, uint64_t* d2h) {
   if (!h) return TV_ERR_INVALID_ARG;
   if (h2d) *h2d = h->host_h2d_bytes;
   if (d2h) *d2h = h->host_d2h_bytes;
-  return TV_OK;
-}
-
-int tv_last_host_read_in_place(tv_handle* h, int* in_place) {
-  if (!h || !in_place) return TV_ERR_INVALID_ARG;
-  *in_place = h->host_in_place;
   return TV_OK;
 }
 
@@ -705,7 +610,6 @@ int tv_destroy(tv_handle* h) {
     cudaFree(h->status);
     if (h->flow_ws) cudaFree(h->flow_ws);
     if (h->stage) cudaFree(h->stage);
-    if (h->small_stage) cudaFree(h->small_stage);
     if (h->lmh_part) cudaFree(h->lmh_part);
     cudaGetLastError();
   }

@@ -12,8 +12,7 @@ typedef void (*any_fn)(void);
 int main(int argc, char** argv) {
   const any_fn entry[] = {
       (any_fn)tv_create,         (any_fn)tv_verify_batch,        (any_fn)tv_verify_batch_debug,
-      (any_fn)tv_verify_batch_host, (any_fn)tv_last_host_copy_bytes,
-      (any_fn)tv_last_host_read_in_place, (any_fn)tv_lm_head,
+      (any_fn)tv_verify_batch_host, (any_fn)tv_last_host_copy_bytes, (any_fn)tv_lm_head,
       (any_fn)tv_draft_children, (any_fn)tv_verify_batch_stats,  (any_fn)tv_get_status,
       (any_fn)tv_destroy,        (any_fn)tv_strerror,            (any_fn)tv_version};
   size_t k;

@@ -335,48 +335,6 @@ def test_host_entry_point_copies_only_needed_draft_rows(tv, shapes):
     assert d2h == B * (R - 1) * 4 + 2 * B * 4
 
 
-@pytest.mark.parametrize("dtype", ["bf16", "fp32"])
-def test_host_entry_point_reads_pinned_rows_in_place(tv, dtype):
-    """Rows in pinned host memory are read in place by the kernels (only the
-    tree arrays and uniforms are copied); the results equal the device path's,
-    and a second call with other inputs on the same handle is not served from
-    anything the first one left behind.  Pageable rows are staged."""
-    name = "eagle_v32k" if dtype == "bf16" else "binary4"
-    B = 24 if dtype == "bf16" else 16
-    w = get_workload(name, batch=B)
-    V = w.vocab
-    v = None
-    for seed in (61, 62):
-        inp = make_inputs(w, seed=seed, device="cuda")
-        R = inp.parents.shape[1]
-        if v is None:
-            v = tv.Verifier(V, R - 1, B, dtype)
-        hp = []
-        for x in (inp.parents, inp.tokens, inp.logits, inp.draft_probs, inp.uniforms):
-            h = torch.empty(x.shape, dtype=x.dtype, pin_memory=True)
-            h.copy_(x)
-            hp.append(h)
-        out = (torch.empty(B, R - 1, dtype=torch.int32), torch.empty(B, dtype=torch.int32),
-               torch.empty(B, dtype=torch.int32))
-        v.verify_host(hp[0], hp[1], hp[2], hp[3], inp.temperature, hp[4], out)
-        assert v.last_host_read_in_place()
-        h2d, d2h = v.last_host_copy_bytes()
-        assert h2d == 2 * B * R * 4 + B * (R + 1) * 4
-        assert d2h == B * (R - 1) * 4 + 2 * B * 4
-        want = v.verify(inp.parents, inp.tokens, inp.logits, inp.draft_probs, inp.temperature,
-                        inp.uniforms)
-        torch.cuda.synchronize()
-        for a, b in zip(out, want):
-            assert torch.equal(a, b.cpu())
-        assert (out[1] >= 0).all()
-    # pageable rows: staged
-    v.verify_host(inp.parents.cpu(), inp.tokens.cpu(), inp.logits.cpu(), inp.draft_probs.cpu(),
-                  inp.temperature, inp.uniforms.cpu(), out)
-    assert not v.last_host_read_in_place()
-    assert v.status() & ~16 == 0
-    v.close()
-
-
 def test_host_argument_errors(tv):
     w = get_workload("tiny", batch=2)
     inp = make_inputs(w, seed=0, device="cuda")
