@@ -115,13 +115,25 @@ GEMM_SOURCES = ["tv_device.cuh", "tv_gemm.cu", "tv_ptx.cuh"]
 DRAFT_SOURCES = ["tv_draft.cu"]
 
 
-def kernel_traffic(workload, batch, kind="persistent"):
-    """DRAM bytes per launch of the dominant kernel (kind "persistent": the
-    verification kernel; "lmhead": the LM-head GEMM) from the committed ncu
-    summary of this workload, or None when there is none or the kernel's
-    sources have changed since it was taken."""
+def kernel_sources_sha256(kind="persistent", root=None):
+    """SHA-256 over name + bytes of the sources of the dominant kernel (kind
+    "persistent": the verification kernel; "lmhead": the LM-head GEMM;
+    "draft": drafting), the key a committed ncu summary is tied to."""
     import hashlib
     sources = {"lmhead": GEMM_SOURCES, "draft": DRAFT_SOURCES}.get(kind, FLOW_SOURCES)
+    h = hashlib.sha256()
+    csrc = os.path.join(root or ROOT, "paper_2505_12398_gb300", "csrc")
+    for name in sources:
+        h.update(name.encode())
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
+def kernel_traffic(workload, batch, kind="persistent"):
+    """DRAM bytes per launch of the dominant kernel from the committed ncu
+    summary of this workload, or None when there is none or the kernel's
+    sources have changed since it was taken."""
     path = os.path.join(ROOT, "profiles", f"launches_{workload}_B{batch}_{kind}.md")
     if not os.path.exists(path):
         return None
@@ -133,13 +145,7 @@ def kernel_traffic(workload, batch, kind="persistent"):
                 fields[key] = val.strip()
     if len(fields) != 2:
         return None
-    h = hashlib.sha256()
-    csrc = os.path.join(ROOT, "paper_2505_12398_gb300", "csrc")
-    for name in sources:
-        h.update(name.encode())
-        with open(os.path.join(csrc, name), "rb") as f:
-            h.update(f.read())
-    if h.hexdigest() != fields["kernel-sources-sha256"]:
+    if kernel_sources_sha256(kind) != fields["kernel-sources-sha256"]:
         return None
     return int(fields["dram-bytes-per-launch"])
 

@@ -55,7 +55,6 @@ using namespace tvk::fused;
 constexpr int kMaxNCW = 8;
 constexpr int kSlots = 3;           // queued slices a CTA holds: one streaming, two ahead
 constexpr int kPBuf = 256;          // partials of a job kept in shared memory by the poll
-constexpr int kMaxSide = 32;        // rows of a normaliser job posted beside a pass
 constexpr unsigned long long kNoPart = ~0ull;   // a partial slot not written yet
 constexpr unsigned kNoTicket = 0xffffffffu;
 constexpr unsigned long long kExitTag = 0x80000000ull;   // tag bit: no more items, exit
@@ -90,9 +89,6 @@ struct Shared {
   Job fjob;                          // a job posted from `ahead`
   float2 pbuf[kPBuf];                // the own job's partials, as read by the poll
   int jkind, jrows, jK, jslice, outstanding;
-  // normalisers of the next sibling's chain, posted beside a pass (side_n = 0: none)
-  int side_n, side_K, side_cnt;
-  int side_rows[kMaxSide];
 };
 
 __device__ __forceinline__ unsigned ld_relaxed_u32(const unsigned* p) {
@@ -763,104 +759,6 @@ __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const
   }
 }
 
-// After posting a pass at node i whose next remaining child c2 has children:
-// once the pass is done the traversal descends into c2's first chain, and the
-// rows of that chain not normalised yet are known now (they do not depend on
-// the pass's S).  Posts their normalisers as a second job of the tree, beside
-// the pass, with partials in rows 1.. of the tree's partial block (the pass
-// uses row 0), so that the descent finds them computed instead of waiting for
-// a normaliser job of its own.  If c2 is removed with rate 0 the rows were
-// read for nothing; the results are the same.
-__device__ void post_side_stats(const TreeSmem& s, Shared& sh, const TravArgs& a,
-                                const FlowArgs& f, int b, int V, int lane, unsigned done) {
-  int n = 0;
-  if (lane == 0 && sh.ctl.job.kind == kJobPass && sh.ctl.pending >= 0) {
-    const int c2 = first_alive_child(s, s.par[sh.ctl.pending]);
-    if (c2 >= 0 && s.first[c2] >= 0) {
-      for (int i = c2; i >= 0; i = first_alive_child(s, i)) {
-        if (s.first[i] < 0) break;
-        if (!(s.rows[i] > 0.f)) {
-          if (n < kMaxSide) sh.side_rows[n] = i;
-          ++n;
-        }
-      }
-    }
-  }
-  n = __shfl_sync(0xffffffffu, n, 0);
-  __syncwarp();
-  if (n == 0 || n > kMaxSide || b == f.withhold_tree) return;
-  const size_t R = (size_t)f.R;
-  const int slice = adaptive_slice(f, V, a.B, true, n, done);
-  const int K = (V + slice - 1) / slice;
-  const int total = n * K;
-  unsigned base = 0u;
-  if (lane == 0) base = atomicAdd(&f.ctr[kCtrTail], (unsigned)total);
-  base = __shfl_sync(0xffffffffu, base, 0);
-  if ((size_t)base + total + kMaxGrid > (size_t)f.cap) {
-    if (lane == 0) raise_abort(a, f);
-    return;
-  }
-  for (int q = lane; q < total; q += 32) {
-    const int r = q / K;
-    __stcg(f.part + ((size_t)b * R + 1 + r) * f.Kmax + (q - r * K), kNoPart);
-  }
-  const int4 w1 = make_int4(kJobStats, slice, 0, 0);
-  for (int q = lane; q < total; q += 32) {
-    const int r = q / K;
-    int4* w = reinterpret_cast<int4*>(f.items + base + q);
-    __stcg(w, make_int4(b, sh.side_rows[r], 1 + r, q - r * K));
-    __stcg(w + 1, w1);
-    __stcg(w + 2, make_int4(0, 0, 0, 0));
-  }
-  fence_gpu();   // bodies and partial resets before the tags
-  __syncwarp();
-  for (int q = lane; q < total; q += 32)
-    st_relaxed_u64(&f.items[base + q].tag, (f.epoch << 32) | (unsigned long long)(base + q));
-  if (lane == 0) {
-    sh.side_n = total;
-    sh.side_K = K;
-    sh.side_cnt = n;
-  }
-}
-
-// The side job's rows: normalisers from their slices (as owner_combine does
-// for a normaliser job), then the float64 M_b^(0) of those rows' children.
-template <typename L>
-__device__ void combine_side_stats(const TravArgs& a, const FlowArgs& f, const TreeSmem& s,
-                                   Shared& sh, int b, int lane) {
-  const int R = a.N + 1, K = sh.side_K, n = sh.side_cnt;
-  const float c_hi = a.c_hi, c_lo = a.c_lo;
-  auto part_of = [&](int r, int k) -> float2 {
-    return unpack_part(__ldcg(f.part + ((size_t)b * R + 1 + r) * f.Kmax + k));
-  };
-  bool bad_row = false;
-  for (int r = lane; r < n; r += 32) {
-    float M = TV_NEG_INF;
-    for (int k2 = 0; k2 < K; ++k2) M = fmaxf(M, part_of(r, k2).x);
-    float S = 0.f;
-    for (int k2 = 0; k2 < K; ++k2) {
-      const float2 pk = part_of(r, k2);
-      if (pk.x != TV_NEG_INF) S += pk.y * L::exp_rel(pk.x, M, c_hi, c_lo);
-    }
-    const int node = sh.side_rows[r];
-    s.rowm[node] = M;
-    s.rows[node] = S;
-    s.invs[node] = 1.0 / (double)S;
-    bad_row |= !(S > 0.f);
-  }
-  if (__any_sync(0xffffffffu, bad_row) && lane == 0) sh.ctl.bad |= 64u;
-  __syncwarp();
-  for (int i = lane + 1; i < R; i += 32) {
-    const int p = s.par[i];
-    bool mine = false;
-    for (int r = 0; r < n; ++r) mine |= (sh.side_rows[r] == p);
-    if (mine) s.mb0[i] = exp2(((double)s.gl[i] - (double)s.rowm[p]) * a.c) * s.invs[p];
-  }
-  __syncwarp();
-  if (lane == 0) sh.side_n = 0;
-  __syncwarp();
-}
-
 // Structure, validation and gathers of tree b; leaves ctl ready to run.
 template <typename L, bool kGiven>
 __device__ void owner_new_tree(const TravArgs& a, const TreeSmem& s, Shared& sh, float* u,
@@ -870,7 +768,6 @@ __device__ void owner_new_tree(const TravArgs& a, const TreeSmem& s, Shared& sh,
   const typename L::elem* logits = reinterpret_cast<const typename L::elem*>(a.logits);
   if (lane == 0) {
     sh.outstanding = 0;
-    sh.side_n = 0;
     sh.ahead.ok = 0;
     Ctl& c = sh.ctl;
     c.bad = 0u;
@@ -1293,30 +1190,6 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
         if (__shfl_sync(0xffffffffu, stop, 0)) break;
         continue;
       }
-      // the normalisers posted beside the job are needed before the next step
-      if (sh.side_n > 0) {
-        const int ns = sh.side_n, Ks = sh.side_K;
-        bool sall = true;
-        for (int q = lane; q < ns; q += 32) {
-          const int r = q / Ks;
-          if (ld_relaxed_u64(f.part + ((size_t)my_tree * R + 1 + r) * f.Kmax + (q - r * Ks)) ==
-              kNoPart)
-            sall = false;
-        }
-        if (!__all_sync(0xffffffffu, sall)) {
-          int stop = 0;
-          if (lane == 0) {
-            if ((++polls & 31u) == 0u && ld_relaxed_u32(&f.ctr[kCtrAbort])) stop = 1;
-            else if (!wait.idle()) {
-              raise_abort(a, f);
-              stop = 1;
-            }
-          }
-          if (__shfl_sync(0xffffffffu, stop, 0)) break;
-          continue;
-        }
-        combine_side_stats<L>(a, f, s, sh, my_tree, lane);
-      }
       wait.reset();
       // after a pass the next job is most often a pass of the same row size:
       // reserve its queue slots now, so that the reservation's round trip
@@ -1395,8 +1268,6 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
             if (a.token_level) sh.ahead.ok = 0;            // (Traversal Verification only)
             else prepare_ahead(s, sh.ctl, sh.ahead, m.mtok2);   // for the job just posted
           }
-          if (!kGiven && !a.token_level)
-            post_side_stats(s, sh, a, f, my_tree, V, lane, __shfl_sync(0xffffffffu, done_est, 0));
           continue;
         }
       }
@@ -1433,8 +1304,6 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
         if (a.token_level) sh.ahead.ok = 0;             // (Traversal Verification only)
         else prepare_ahead(s, sh.ctl, sh.ahead, m.mtok2);    // while this job runs
       }
-      if (!kGiven && !a.token_level)
-        post_side_stats(s, sh, a, f, my_tree, V, lane, __shfl_sync(0xffffffffu, done_est, 0));
     }
   }
 }

@@ -45,19 +45,18 @@ def _copy_tree(tmp_path):
 
 
 def test_kernel_traffic_follows_the_source_hash(tmp_path, monkeypatch):
-    prof = os.path.join(bench.ROOT, "profiles", "launches_eagle_v128k_B128_persistent.md")
-    if not os.path.exists(prof):
-        pytest.skip("no committed launch profile")
+    """A profile's DRAM figure is used only while the kernel sources hash to
+    the value recorded with it."""
     root = _copy_tree(tmp_path)
     monkeypatch.setattr(bench, "ROOT", str(root))
-    got = bench.kernel_traffic("eagle_v128k", 128)
-    if got is None:
-        pytest.skip("the committed profile predates the current kernel sources")
-    assert got > 0
-    assert bench.kernel_traffic("eagle_v128k", 64) is None   # no profile of that batch
+    prof = root / "profiles" / "launches_testload_B7_persistent.md"
+    prof.write_text("# test\n\n    kernel-sources-sha256: "
+                    + bench.kernel_sources_sha256() + "\n    dram-bytes-per-launch: 12345\n")
+    assert bench.kernel_traffic("testload", 7) == 12345
+    assert bench.kernel_traffic("testload", 8) is None   # no profile of that batch
     src = root / "paper_2505_12398_gb300" / "csrc" / "tv_flow.cu"
     src.write_text(src.read_text() + "\n// changed\n")
-    assert bench.kernel_traffic("eagle_v128k", 128) is None
+    assert bench.kernel_traffic("testload", 7) is None
 
 
 def test_lmhead_oracle_leg_matches_the_oracle_on_the_generated_logits(tmp_path):
