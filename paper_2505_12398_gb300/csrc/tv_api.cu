@@ -62,7 +62,8 @@ constexpr unsigned kPathFlags = TV_FLAG_UNFUSED | TV_FLAG_CLUSTER | TV_FLAG_PERS
 enum Path { kPathThree = 0, kPathCluster = 1, kPathPersistent = 2 };
 
 FlowPlan flow_plan(const tv_handle* h, int R, int B) {
-  return tv_flow_plan(R, B, h->smem_per_sm, h->smem_per_block, h->flow_force[0], h->flow_force[1],
+  return tv_flow_plan(R, B, h->vocab, h->smem_per_sm, h->smem_per_block, h->flow_force[0],
+                      h->flow_force[1],
                       h->flow_force[2], h->flow_force[3], h->flow_force[4]);
 }
 

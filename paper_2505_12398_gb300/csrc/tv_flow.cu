@@ -1448,7 +1448,7 @@ int tv_flow_bind(void* base, size_t bytes, int B, int R, int V, const FlowPlan& 
   return (size_t)(p - static_cast<char*>(base)) <= bytes ? 0 : -4;
 }
 
-FlowPlan tv_flow_plan(int R, int B, int smem_per_sm, int smem_per_block, int force_ncw,
+FlowPlan tv_flow_plan(int R, int B, int V, int smem_per_sm, int smem_per_block, int force_ncw,
                       int force_stages, int force_slice_pass, int force_slice_stats,
                       int force_slice_min) {
   FlowPlan p;
@@ -1456,9 +1456,15 @@ FlowPlan tv_flow_plan(int R, int B, int smem_per_sm, int smem_per_block, int for
   // every CTA is busy anyway, and larger slices mean fewer queue items,
   // partials and combines per byte (at 1024 trees of 128256 tokens, 32768-
   // token slices stream 14 % faster than 8192; at 128 trees, where a job's
-  // latency sets the time, 8192 is best)
-  p.slice_pass = B >= 1024 ? 32768 : (B >= 256 ? 16384 : 8192);
-  p.slice_stats = B >= 256 ? 32768 : 16384;
+  // latency sets the time, 8192 is best).  From 1024 trees a pass takes a
+  // quarter row per slice and a normaliser half a row when that is larger
+  // (V = 151936: 38144 and 76032 tokens, 4 % faster than 32768 for both; V =
+  // 128256: 64256-token normaliser slices, 4 % faster)
+  auto tiles_up = [](long long x) { return (int)((x + 255) / 256 * 256); };
+  p.slice_pass = B >= 1024 ? std::max(32768, tiles_up((V + 3LL) / 4))
+                           : (B >= 256 ? 16384 : 8192);
+  p.slice_stats = B >= 1024 ? std::max(32768, tiles_up((V + 1LL) / 2))
+                            : (B >= 256 ? 32768 : 16384);
   if (force_ncw == 4 || force_ncw == 8) p.ncw = force_ncw;
   if (force_slice_pass >= 256 && force_slice_pass % 256 == 0) p.slice_pass = force_slice_pass;
   if (force_slice_stats >= 256 && force_slice_stats % 256 == 0) p.slice_stats = force_slice_stats;

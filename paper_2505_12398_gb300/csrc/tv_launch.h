@@ -100,7 +100,7 @@ struct FlowPlan {
 };
 
 // Default plan for R = N+1 rows and B trees (tuning overrides: force_* > 0).
-FlowPlan tv_flow_plan(int R, int B, int smem_per_sm, int smem_per_block, int force_ncw,
+FlowPlan tv_flow_plan(int R, int B, int V, int smem_per_sm, int smem_per_block, int force_ncw,
                       int force_stages, int force_slice_pass, int force_slice_stats,
                       int force_slice_min);
 // Workspace for slices of at least `min_slice` tokens.

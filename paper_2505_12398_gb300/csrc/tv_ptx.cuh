@@ -1,9 +1,9 @@
 // tv_ptx.cuh -- inline-PTX wrappers: mbarriers, 1-D TMA bulk copies, named
 // barriers and distributed shared memory inside a thread-block cluster.
 //
-// Every wait is bounded, in tries and in time: try_wait is polled at most
-// kSpinLimit times and for at most kWaitLimitNs, and the caller turns a
-// timeout into an error status instead of hanging the GPU.
+// Every wait is bounded: try_wait is polled at most kSpinLimit times, each
+// try suspending at most kTrySuspendNs, and the caller turns a timeout into an
+// error status instead of hanging the GPU.
 #pragma once
 
 #include <cuda_runtime.h>
@@ -37,62 +37,40 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
 
+// Longest time one try_wait may suspend the thread before it reports "not
+// yet" (the suspend-time hint, in nanoseconds): kSpinLimit tries then last at
+// most about kSpinLimit * kTrySuspendNs (~2 s).
+constexpr uint32_t kTrySuspendNs = 2000u;
+
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
+      : "r"(smem_u32(bar)), "r"(parity), "n"(kTrySuspendNs)
       : "memory");
   return ok != 0;
 }
 
-// Nanoseconds of the global timer.
-__device__ __forceinline__ uint64_t ptx_global_ns() {
-  uint64_t t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-
-// A try_wait may suspend the thread for a system-dependent time before it
-// reports "not yet", so an iteration count alone does not bound the wait in
-// time: every 64 failed tries also compare the global timer against
-// kWaitLimitNs.
-constexpr uint64_t kWaitLimitNs = 2000000000ull;
-
-// Waits until the phase with the given parity has completed; false on timeout
-// (kSpinLimit tries or kWaitLimitNs, whichever comes first).
+// Waits until the phase with the given parity has completed; false on timeout.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
-  uint64_t t0 = 0;
-  for (uint32_t i = 0; i < kSpinLimit; ++i) {
+  for (uint32_t i = 0; i < kSpinLimit; ++i)
     if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 63u) == 63u) {
-      const uint64_t now = ptx_global_ns();
-      if (t0 == 0) t0 = now;
-      else if (now - t0 > kWaitLimitNs) return false;
-    }
-  }
   return false;
 }
 
 // Same wait with cluster-scope acquire (for arrivals made by peer CTAs).
 __device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity) {
-  uint64_t t0 = 0;
   for (uint32_t i = 0; i < kSpinLimit; ++i) {
-    if ((i & 63u) == 63u) {
-      const uint64_t now = ptx_global_ns();
-      if (t0 == 0) t0 = now;
-      else if (now - t0 > kWaitLimitNs) return false;
-    }
     uint32_t ok;
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
         "selp.u32 %0, 1, 0, p;\n\t}"
         : "=r"(ok)
-        : "r"(smem_u32(bar)), "r"(parity)
+        : "r"(smem_u32(bar)), "r"(parity), "n"(kTrySuspendNs)
         : "memory");
     if (ok) return true;
   }
