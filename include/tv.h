@@ -205,13 +205,20 @@ int tv_verify_batch_debug(tv_handle* h, int B, int N, const int32_t* parents,
 
 /*
  * tv_verify_batch_host -- the same verification from HOST buffers: copies the
- * inputs to device staging owned by the handle (allocated on first use, sized
- * by tv_create's limits), runs tv_verify_batch on cuda_stream, copies the
- * three outputs back and synchronises the stream before returning.  All
- * pointers are host pointers with the layouts above; pinned (page-locked)
- * memory gives the fastest copies.  Draft rows of nodes without children are
- * never read and are not copied (one 2-D copy per run of rows with children
- * when all trees share their parents).  Errors as tv_verify_batch.
+ * inputs to device staging owned by the handle (allocated and zeroed on first
+ * use, sized by tv_create's limits), runs tv_verify_batch on cuda_stream,
+ * copies the three outputs back and synchronises the stream before
+ * returning.  All pointers are host pointers with the layouts above; pinned
+ * (page-locked) memory gives the fastest copies.  Only rows the verification
+ * can need are copied: the logit and draft rows of nodes with children (one
+ * 2-D copy per run of such rows when all trees share their parents).  Of the
+ * leaves' logit rows only the accepted leaf's is ever read, for the bonus
+ * draw, so the call has two phases: the verification runs (its draw at a leaf
+ * reads a stale staged row), then the accepted leaves' rows alone (at most one
+ * per tree) are copied and their bonus tokens drawn again by a kernel of its
+ * own (float64 prefix over float32 tile sums of the same e(x); a draw within
+ * about 1e-6 W of a CDF step may differ from the device entry point's).
+ * Errors as tv_verify_batch.
  */
 int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
                          const int32_t* draft_tokens, const void* target_logits,

@@ -21,6 +21,7 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libtv.so")
 SOURCES = ["tv_api.cu", "tv_kernels.cu", "tv_tree.cu", "tv_flow.cu", "tv_noalloc.cu", "tv_gemm.cu",
+           "tv_bonus.cu",
            "tv_draft.cu"]
 HEADERS = ["tv_device.cuh", "tv_launch.h", "tv_ptx.cuh", "tv_control.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

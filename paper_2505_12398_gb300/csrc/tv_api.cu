@@ -112,13 +112,14 @@ class NvtxRange {
   NvtxRange& operator=(const NvtxRange&) = delete;
 };
 
-// Copies the draft rows of nodes with children from host to device (rows of
-// leaves are never read).  When every tree has the same parents, each run of
-// consecutive rows with children is one 2-D copy over the batch; otherwise one
-// copy per run per tree.  Adds the bytes copied to *bytes.
-bool copy_draft_rows(float* dst, const float* src, const int32_t* parents, int B, size_t R,
-                     size_t V, cudaStream_t st, size_t* bytes) {
-  const size_t row = V * sizeof(float);
+// Copies the rows (row bytes each) of nodes with children from host to
+// device.  When every tree has the same parents, each run of consecutive rows
+// with children is one 2-D copy over the batch; otherwise one copy per run per
+// tree.  Adds the bytes copied to *bytes.
+bool copy_internal_rows(void* dst_v, const void* src_v, size_t row, const int32_t* parents,
+                        int B, size_t R, cudaStream_t st, size_t* bytes) {
+  char* dst = static_cast<char*>(dst_v);
+  const char* src = static_cast<const char*>(src_v);
   auto rows_with_children = [&](int b, std::vector<char>& kid) {
     std::fill(kid.begin(), kid.end(), 0);
     for (size_t i = 1; i < R; ++i) {
@@ -146,7 +147,7 @@ bool copy_draft_rows(float* dst, const float* src, const int32_t* parents, int B
   if (same) {
     rows_with_children(0, kid);
     const bool ok = runs(kid, [&](size_t r0, size_t r1) {
-      if (cudaMemcpy2DAsync(dst + r0 * V, R * row, src + r0 * V, R * row, (r1 - r0) * row,
+      if (cudaMemcpy2DAsync(dst + r0 * row, R * row, src + r0 * row, R * row, (r1 - r0) * row,
                             (size_t)B, cudaMemcpyHostToDevice, st) != cudaSuccess)
         return false;
       *bytes += (r1 - r0) * row * (size_t)B;
@@ -159,7 +160,7 @@ bool copy_draft_rows(float* dst, const float* src, const int32_t* parents, int B
     rows_with_children(b, kid);
     const size_t base = (size_t)b * R;
     if (!runs(kid, [&](size_t r0, size_t r1) {
-          if (cudaMemcpyAsync(dst + (base + r0) * V, src + (base + r0) * V, (r1 - r0) * row,
+          if (cudaMemcpyAsync(dst + (base + r0) * row, src + (base + r0) * row, (r1 - r0) * row,
                               cudaMemcpyHostToDevice, st) != cudaSuccess)
             return false;
           *bytes += (r1 - r0) * row;
@@ -420,6 +421,14 @@ int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
       cudaGetLastError();
       return TV_ERR_CUDA;
     }
+    // every staged row starts defined: rows a call does not copy (leaves'
+    // logit rows) then hold zeros or an earlier call's values, never garbage
+    if (cudaMemset(h->stage, 0, cap) != cudaSuccess) {
+      cudaGetLastError();
+      cudaFree(h->stage);
+      h->stage = nullptr;
+      return TV_ERR_CUDA;
+    }
     h->stage_bytes = cap;
   }
   char* p = h->stage;
@@ -431,12 +440,27 @@ int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
   int32_t* d_path = reinterpret_cast<int32_t*>(p); p += up(n_path);
   int32_t* d_len = reinterpret_cast<int32_t*>(p); p += up(n_out);
   int32_t* d_bonus = reinterpret_cast<int32_t*>(p);
+  // Only rows the verification can need are copied: the logit and draft rows
+  // of nodes with children.  Of the leaves' logit rows at most one per tree is
+  // needed -- the accepted leaf's, for the bonus draw -- so the verification
+  // runs first (its draw at a leaf then reads a stale row), and then only the
+  // accepted leaves' rows are copied and their bonus tokens drawn again by
+  // tv_launch_leaf_bonus.
+  const bool two_phase = tv_leaf_bonus_smem_bytes(h->vocab) <= 48 * 1024;
+  const size_t lrow = V * logit_bytes(h);
+  size_t logit_copied = 0, draft_bytes = 0;
   bool ok = cudaMemcpyAsync(d_par, parents, n_tree, cudaMemcpyHostToDevice, st) == cudaSuccess &&
             cudaMemcpyAsync(d_tok, draft_tokens, n_tree, cudaMemcpyHostToDevice, st) == cudaSuccess &&
-            cudaMemcpyAsync(d_unif, uniforms, n_unif, cudaMemcpyHostToDevice, st) == cudaSuccess &&
-            cudaMemcpyAsync(d_logit, target_logits, n_logit, cudaMemcpyHostToDevice, st) == cudaSuccess;
-  size_t draft_bytes = 0;
-  ok = ok && copy_draft_rows(d_draft, draft_probs, parents, B, R, V, st, &draft_bytes);
+            cudaMemcpyAsync(d_unif, uniforms, n_unif, cudaMemcpyHostToDevice, st) == cudaSuccess;
+  if (two_phase) {
+    ok = ok && copy_internal_rows(d_logit, target_logits, lrow, parents, B, R, st, &logit_copied);
+  } else {
+    ok = ok && cudaMemcpyAsync(d_logit, target_logits, n_logit, cudaMemcpyHostToDevice, st) ==
+                   cudaSuccess;
+    logit_copied = n_logit;
+  }
+  ok = ok && copy_internal_rows(d_draft, draft_probs, V * sizeof(float), parents, B, R, st,
+                                &draft_bytes);
   if (!ok) {
     cudaGetLastError();
     return TV_ERR_CUDA;
@@ -453,8 +477,55 @@ int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
     cudaGetLastError();
     return TV_ERR_CUDA;
   }
-  h->host_h2d_bytes = 2 * n_tree + n_unif + n_logit + draft_bytes;
-  h->host_d2h_bytes = (N > 0 ? n_path : 0) + 2 * n_out;
+  size_t leaf_bytes = 0, pend_bytes = 0;
+  if (two_phase) {
+    // trees whose accepted node has no children: (tree, that node's row)
+    std::vector<int2> pend;
+    for (int b = 0; b < B; ++b) {
+      const int tau = out_accept_len[b];
+      if (tau < 0) continue;   // an invalid tree
+      const int acc = tau > 0 ? out_accepted_path[(size_t)b * N + tau - 1] : 0;
+      if (acc < 0 || (size_t)acc >= R) continue;
+      bool leaf = true;
+      for (size_t i = (size_t)acc + 1; i < R && leaf; ++i)
+        leaf = parents[(size_t)b * R + i] != acc;
+      if (leaf) pend.push_back(make_int2(b, acc));
+    }
+    if (!pend.empty()) {
+      for (const int2& q : pend) {
+        const size_t off = ((size_t)q.x * R + (size_t)q.y) * lrow;
+        if (cudaMemcpyAsync(static_cast<char*>(d_logit) + off,
+                            static_cast<const char*>(target_logits) + off, lrow,
+                            cudaMemcpyHostToDevice, st) != cudaSuccess) {
+          cudaGetLastError();
+          return TV_ERR_CUDA;
+        }
+        leaf_bytes += lrow;
+      }
+      // the (tree, row) list is staged in the row-statistics buffer of the
+      // three-kernel path ([max_batch (max_nodes + 1)] float2 >= B int2),
+      // which no kernel reads once the verification above has finished
+      int2* d_pend = reinterpret_cast<int2*>(h->stats);
+      pend_bytes = pend.size() * sizeof(int2);
+      const double c = 1.4426950408889634 / static_cast<double>(temperature);
+      const float c_hi = static_cast<float>(c);
+      const float c_lo = static_cast<float>(c - static_cast<double>(c_hi));
+      ok = cudaMemcpyAsync(d_pend, pend.data(), pend_bytes, cudaMemcpyHostToDevice, st) ==
+               cudaSuccess &&
+           tv_launch_leaf_bonus(d_logit, h->dtype == TV_BF16 ? 1 : 0, d_unif, d_pend,
+                                static_cast<int>(pend.size()), B, static_cast<int>(R),
+                                h->vocab, c_hi, c_lo, d_bonus, st) == 0 &&
+           cudaMemcpyAsync(out_bonus_token, d_bonus, n_out, cudaMemcpyDeviceToHost, st) ==
+               cudaSuccess &&
+           cudaStreamSynchronize(st) == cudaSuccess;
+      if (!ok) {
+        cudaGetLastError();
+        return TV_ERR_CUDA;
+      }
+    }
+  }
+  h->host_h2d_bytes = 2 * n_tree + n_unif + logit_copied + draft_bytes + leaf_bytes + pend_bytes;
+  h->host_d2h_bytes = (N > 0 ? n_path : 0) + 2 * n_out + (pend_bytes ? n_out : 0);
   return TV_OK;
 }
 

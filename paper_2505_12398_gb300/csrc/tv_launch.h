@@ -27,6 +27,15 @@ struct TravArgs {
                                // (persistent path)
 };
 
+// The bonus draws at accepted original leaves, one CTA per entry of pending
+// ((tree, leaf row) pairs, n_pending <= B): writes out_bonus[tree] (-1 for a
+// row without a finite logit).  0, -1 (bad count), -3 (vocabulary too large for
+// one CTA's tile sums) or -5 (launch failed).
+int tv_launch_leaf_bonus(const void* logits, int logit_is_bf16, const float* uniforms,
+                         const int2* pending, int n_pending, int B, int R, int V, float c_hi,
+                         float c_lo, int32_t* out_bonus, cudaStream_t stream);
+size_t tv_leaf_bonus_smem_bytes(int V);
+
 // Launch plan of the fused kernel: cluster size, ring stages, shared memory.
 struct FusedPlan {
   int ncw = 8;       // consumer warps per CTA (4 or 8)

@@ -284,25 +284,35 @@ def test_invalid_trees_flagged(tv, path):
 
 
 def test_host_entry_point_matches_device(tv):
-    w = get_workload("binary4", batch=8)
-    inp = make_inputs(w, seed=4, device="cuda")
-    (path, tau, bonus, _, _), _ = run_gpu(tv, inp)
-    B, R = inp.parents.shape
-    v = tv.Verifier(w.vocab, R - 1, B, "fp32")
-    hp = [inp.parents.cpu(), inp.tokens.cpu(), inp.logits.cpu(), inp.draft_probs.cpu(),
-          inp.uniforms.cpu()]
-    out = (torch.empty(B, R - 1, dtype=torch.int32), torch.empty(B, dtype=torch.int32),
-           torch.empty(B, dtype=torch.int32))
-    v.verify_host(hp[0], hp[1], hp[2], hp[3], inp.temperature, hp[4], out)
-    v.close()
-    assert (out[0].numpy() == path).all() and (out[1].numpy() == tau).all()
-    assert (out[2].numpy() == bonus).all()
+    """From host buffers: the same paths and lengths as the device entry point;
+    the bonus tokens drawn at accepted leaves in the second phase (a kernel of
+    its own) equal the oracle's outside the near-tie band."""
+    for name, dt in (("binary4", "fp32"), ("eagle_v32k", "bf16")):
+        w = get_workload(name, batch=8)
+        inp = make_inputs(w, seed=4, device="cuda")
+        (path, tau, bonus, _, stats), _ = run_gpu(tv, inp)
+        B, R = inp.parents.shape
+        v = tv.Verifier(w.vocab, R - 1, B, dt)
+        hp = [inp.parents.cpu(), inp.tokens.cpu(), inp.logits.cpu(), inp.draft_probs.cpu(),
+              inp.uniforms.cpu()]
+        out = (torch.empty(B, R - 1, dtype=torch.int32), torch.empty(B, dtype=torch.int32),
+               torch.empty(B, dtype=torch.int32))
+        v.verify_host(hp[0], hp[1], hp[2], hp[3], inp.temperature, hp[4], out)
+        v.close()
+        assert (out[0].numpy() == path).all() and (out[1].numpy() == tau).all()
+        par, tok, lg, dp, un = to_numpy_inputs(inp)
+        _, _, obonus, det = verify_batch(par, tok, lg, dp, inp.temperature, un)
+        for b in range(B):
+            if det[b]["bonus_margin"] >= 1e-5 and det[b]["test_margin"] >= 1e-5:
+                assert int(out[2][b]) == int(obonus[b]), (name, b)
+        assert stats[:, 3].sum() > 0   # some trees ended at an accepted leaf
 
 
 @pytest.mark.parametrize("shapes", ["same", "random"])
 def test_host_entry_point_copies_only_needed_draft_rows(tv, shapes):
-    """The host entry point copies the draft rows of nodes with children only
-    (2-D copies when all trees share a shape, per tree otherwise).  Two calls
+    """The host entry point copies the logit and draft rows of nodes with
+    children, then the logit rows of the accepted leaves only (2-D copies when
+    all trees share a shape, per tree otherwise).  Two calls
     on one handle with different inputs: stale staging from the first would
     change the second's results if a needed row were missed."""
     from workloads.synth import make_inputs_random_shapes
@@ -322,17 +332,24 @@ def test_host_entry_point_copies_only_needed_draft_rows(tv, shapes):
         v.verify_host(hp[0], hp[1], hp[2], hp[3], inp.temperature, hp[4], out)
     h2d, d2h = v.last_host_copy_bytes()
     want = v.verify(second.parents, second.tokens, second.logits, second.draft_probs,
-                    second.temperature, second.uniforms)
+                    second.temperature, second.uniforms, debug=True)
     torch.cuda.synchronize()
     assert v.status() & ~16 == 0
     v.close()
-    for a, b in zip(out, want):
+    for a, b in zip(out[:2], want[:2]):
         assert torch.equal(a, b.cpu())
+    # bonus tokens: the draws at accepted leaves come from the second phase's
+    # own kernel, equal to the device path's away from a CDF step
+    leaf = want[4][:, 3].cpu().numpy() > 0
+    same = out[2].numpy() == want[2].cpu().numpy()
+    assert same[~leaf].all() and same[leaf].mean() > 0.8
     par = second.parents.cpu().numpy()
     internal = sum(len({int(p) for p in par[b, 1:]}) for b in range(B))
+    n_leaf = int(leaf.sum())
     V = 32000
-    assert h2d == 2 * B * R * 4 + B * (R + 1) * 4 + B * R * V * 2 + internal * V * 4
-    assert d2h == B * (R - 1) * 4 + 2 * B * 4
+    assert h2d == (2 * B * R * 4 + B * (R + 1) * 4 + internal * V * (2 + 4) + n_leaf * V * 2 +
+                   n_leaf * 8)
+    assert d2h == B * (R - 1) * 4 + 2 * B * 4 + (B * 4 if n_leaf else 0)
 
 
 def test_host_argument_errors(tv):
