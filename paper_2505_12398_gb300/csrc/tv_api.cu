@@ -51,6 +51,11 @@ struct tv_handle {
   bool timing = false;
   bool timed_call = false;
   cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
+  // tv_verify_batch_host: two copy streams (a 2-D host-to-device copy on one
+  // stream reaches about 60 % of the link; split over two it saturates it)
+  // and the events that order them against the caller's stream
+  cudaStream_t copy_st[2] = {nullptr, nullptr};
+  cudaEvent_t copy_ev[3] = {nullptr, nullptr, nullptr};
 };
 
 namespace {
@@ -117,7 +122,7 @@ class NvtxRange {
 // with children is one 2-D copy over the batch; otherwise one copy per run per
 // tree.  Adds the bytes copied to *bytes.
 bool copy_internal_rows(void* dst_v, const void* src_v, size_t row, const int32_t* parents,
-                        int B, size_t R, cudaStream_t st, size_t* bytes) {
+                        int B, size_t R, const cudaStream_t* sts, int n_st, size_t* bytes) {
   char* dst = static_cast<char*>(dst_v);
   const char* src = static_cast<const char*>(src_v);
   auto rows_with_children = [&](int b, std::vector<char>& kid) {
@@ -147,9 +152,15 @@ bool copy_internal_rows(void* dst_v, const void* src_v, size_t row, const int32_
   if (same) {
     rows_with_children(0, kid);
     const bool ok = runs(kid, [&](size_t r0, size_t r1) {
-      if (cudaMemcpy2DAsync(dst + r0 * row, R * row, src + r0 * row, R * row, (r1 - r0) * row,
-                            (size_t)B, cudaMemcpyHostToDevice, st) != cudaSuccess)
-        return false;
+      // the batch split between the streams, one 2-D copy each
+      for (int k = 0; k < n_st; ++k) {
+        const size_t b0 = (size_t)B * k / n_st, b1 = (size_t)B * (k + 1) / n_st;
+        if (b1 == b0) continue;
+        if (cudaMemcpy2DAsync(dst + (b0 * R + r0) * row, R * row, src + (b0 * R + r0) * row,
+                              R * row, (r1 - r0) * row, b1 - b0, cudaMemcpyHostToDevice,
+                              sts[k]) != cudaSuccess)
+          return false;
+      }
       *bytes += (r1 - r0) * row * (size_t)B;
       return true;
     });
@@ -161,7 +172,7 @@ bool copy_internal_rows(void* dst_v, const void* src_v, size_t row, const int32_
     const size_t base = (size_t)b * R;
     if (!runs(kid, [&](size_t r0, size_t r1) {
           if (cudaMemcpyAsync(dst + (base + r0) * row, src + (base + r0) * row, (r1 - r0) * row,
-                              cudaMemcpyHostToDevice, st) != cudaSuccess)
+                              cudaMemcpyHostToDevice, sts[b % n_st]) != cudaSuccess)
             return false;
           *bytes += (r1 - r0) * row;
           return true;
@@ -452,15 +463,31 @@ int tv_verify_batch_host(tv_handle* h, int B, int N, const int32_t* parents,
   bool ok = cudaMemcpyAsync(d_par, parents, n_tree, cudaMemcpyHostToDevice, st) == cudaSuccess &&
             cudaMemcpyAsync(d_tok, draft_tokens, n_tree, cudaMemcpyHostToDevice, st) == cudaSuccess &&
             cudaMemcpyAsync(d_unif, uniforms, n_unif, cudaMemcpyHostToDevice, st) == cudaSuccess;
+  // the row copies run on the handle's two copy streams, after everything
+  // queued on st so far and before the verification that follows on st
+  if (!h->copy_st[0]) {
+    for (int k = 0; k < 2; ++k)
+      ok = ok && cudaStreamCreateWithFlags(&h->copy_st[k], cudaStreamNonBlocking) == cudaSuccess;
+    for (int k = 0; k < 3; ++k)
+      ok = ok && cudaEventCreateWithFlags(&h->copy_ev[k], cudaEventDisableTiming) == cudaSuccess;
+  }
+  ok = ok && cudaEventRecord(h->copy_ev[0], st) == cudaSuccess &&
+       cudaStreamWaitEvent(h->copy_st[0], h->copy_ev[0], 0) == cudaSuccess &&
+       cudaStreamWaitEvent(h->copy_st[1], h->copy_ev[0], 0) == cudaSuccess;
   if (two_phase) {
-    ok = ok && copy_internal_rows(d_logit, target_logits, lrow, parents, B, R, st, &logit_copied);
+    ok = ok && copy_internal_rows(d_logit, target_logits, lrow, parents, B, R, h->copy_st, 2,
+                                  &logit_copied);
   } else {
     ok = ok && cudaMemcpyAsync(d_logit, target_logits, n_logit, cudaMemcpyHostToDevice, st) ==
                    cudaSuccess;
     logit_copied = n_logit;
   }
-  ok = ok && copy_internal_rows(d_draft, draft_probs, V * sizeof(float), parents, B, R, st,
-                                &draft_bytes);
+  ok = ok && copy_internal_rows(d_draft, draft_probs, V * sizeof(float), parents, B, R,
+                                h->copy_st, 2, &draft_bytes);
+  ok = ok && cudaEventRecord(h->copy_ev[1], h->copy_st[0]) == cudaSuccess &&
+       cudaEventRecord(h->copy_ev[2], h->copy_st[1]) == cudaSuccess &&
+       cudaStreamWaitEvent(st, h->copy_ev[1], 0) == cudaSuccess &&
+       cudaStreamWaitEvent(st, h->copy_ev[2], 0) == cudaSuccess;
   if (!ok) {
     cudaGetLastError();
     return TV_ERR_CUDA;
@@ -676,6 +703,10 @@ int tv_destroy(tv_handle* h) {
     if (guard.ok()) cudaDeviceSynchronize();
     for (int k = 0; k < 4; ++k)
       if (h->ev[k]) cudaEventDestroy(h->ev[k]);
+    for (int k = 0; k < 2; ++k)
+      if (h->copy_st[k]) cudaStreamDestroy(h->copy_st[k]);
+    for (int k = 0; k < 3; ++k)
+      if (h->copy_ev[k]) cudaEventDestroy(h->copy_ev[k]);
     cudaFree(h->row_list);
     cudaFree(h->n_rows);
     cudaFree(h->stats);
