@@ -73,10 +73,13 @@ enum {
 };
 
 /* Flags for tv_create.  At most one path flag may be given; with none the
-   library picks the path (the persistent kernel when V % 8 == 0, else the three-kernel
-   path).  All paths compute the same results; the two single-kernel paths read
-   rows with bulk copies and need V % 8 == 0, other vocabularies always take
-   the three-kernel path. */
+   library picks the path: when V % 8 == 0, the cluster-per-tree kernel for
+   V <= 49152 and N + 1 <= 128 (short rows, where one cluster per tree is
+   faster than publishing every job through the persistent kernel's queue;
+   calls with given row normalisers still run the persistent kernel), else the
+   persistent kernel; the three-kernel path otherwise.  All paths compute the
+   same results; the two single-kernel paths read rows with bulk copies and
+   need V % 8 == 0, other vocabularies always take the three-kernel path. */
 enum {
   TV_FLAG_NONE = 0u,
   /* Three kernels: row normalisers of every internal row, then one CTA per
@@ -295,8 +298,9 @@ int tv_draft_children(tv_handle* h, int B, int N, const int32_t* parents,
  * temperature), so no row is streamed to normalise it.  out_node_p and
  * out_stats are optional (NULL) and have the layouts of tv_verify_batch_debug
  * (out_stats[b][4], rows normalised by this call, is then 0).  Runs on the
- * persistent kernel only: other paths, and calls on a capturing stream, return
- * TV_ERR_INVALID_ARG.
+ * persistent kernel only (a handle that picks its path itself uses it here
+ * for every V): handles created for the other paths, and calls on a
+ * capturing stream, return TV_ERR_INVALID_ARG.
  * Errors: those of tv_verify_batch.
  */
 int tv_verify_batch_stats(tv_handle* h, int B, int N, const int32_t* parents,

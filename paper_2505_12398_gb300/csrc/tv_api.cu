@@ -78,6 +78,11 @@ int flow_min_slice(const tv_handle* h) {
   return p.slice_min;
 }
 
+// Largest vocabulary and tree for which a handle that chose its path itself
+// takes the cluster path rather than the persistent kernel.
+constexpr int kClusterMaxVocab = 49152;
+constexpr int kClusterMaxRows = 128;
+
 Path choose_path(const tv_handle* h, int B, int R, FusedPlan* plan) {
   if ((h->vocab % 8) != 0 || (h->flags & TV_FLAG_UNFUSED)) return kPathThree;
   if (h->flags & TV_FLAG_CLUSTER) {
@@ -86,6 +91,16 @@ Path choose_path(const tv_handle* h, int B, int R, FusedPlan* plan) {
     return plan->ok ? kPathCluster : kPathThree;
   }
   if (!h->flow_ws || !flow_plan(h, R, B).ok) return kPathThree;
+  if (!(h->flags & TV_FLAG_PERSISTENT) && h->vocab <= kClusterMaxVocab && R <= kClusterMaxRows) {
+    // short rows: a job of the persistent kernel costs more to publish and
+    // combine through its global queue than to stream, and one cluster per
+    // tree, exchanging partials through distributed shared memory, is faster
+    // (V = 32000, EAGLE-shaped trees: 13-22 % less time at 16 to 2048 trees;
+    // the persistent kernel is faster from V = 128256 and on deep trees)
+    *plan = tv_fused_plan(B, R, h->vocab, h->sm_count, h->smem_per_sm, h->smem_per_block,
+                          h->force_ncw, h->force_c, h->force_stages);
+    if (plan->ok) return kPathCluster;
+  }
   return kPathPersistent;
 }
 
@@ -261,6 +276,11 @@ int verify_impl(tv_handle* h, int B, int N, const int32_t* parents, const int32_
                          h->force_ncw, h->force_c, h->force_stages);
     path = plan.ok ? kPathCluster : kPathThree;
   }
+  // given row normalisers are read by the persistent kernel only: a handle
+  // that chose the cluster path itself runs them there
+  if (row_stats && path == kPathCluster && !(h->flags & TV_FLAG_CLUSTER) && h->flow_ws &&
+      flow_plan(h, N + 1, B).ok)
+    path = kPathPersistent;
   // the three-kernel path implements Traversal Verification only
   if (path == kPathThree && a.token_level) return TV_ERR_INVALID_ARG;
   // given row normalisers are read by the persistent kernel only

@@ -28,7 +28,7 @@ def tv():
     return tv
 
 
-def z_counts(tv, shape, V, count, seed, wrong_target=False, method="traversal"):
+def z_counts(tv, shape, V, count, seed, wrong_target=False, method="traversal", path="auto"):
     rng = np.random.default_rng(seed)
     L = 4
     tb = float_table(V, L, seed, concentration=0.8)
@@ -55,7 +55,7 @@ def z_counts(tv, shape, V, count, seed, wrong_target=False, method="traversal"):
     dp = torch.from_numpy(drafts).to(dev)
     un = torch.rand(count, n + 1, generator=torch.Generator(device=dev).manual_seed(seed),
                     device=dev)
-    v = tv.Verifier(V, n - 1, count, "fp32", method=method)
+    v = tv.Verifier(V, n - 1, count, "fp32", method=method, path=path)
     path, tau, bonus = v.verify(par, tok, lg, dp, 1.0, un)
     torch.cuda.synchronize()
     status = v.status()
@@ -91,11 +91,14 @@ def chi2_p(obs, exp):
     return scipy.stats.chisquare(o, e).pvalue
 
 
-@pytest.mark.parametrize("shape,V", [([-1, 0, 0, 1, 1, 2, 2], 4),
-                                     ([-1, 0, 0, 0, 1, 1, 2, 4], 3),
-                                     ([-1, 0, 1, 2], 8)])
-def test_kernel_output_law_is_target(tv, shape, V):
-    obs, exp = z_counts(tv, shape, V, 1_000_000, seed=V * 17 + len(shape))
+@pytest.mark.parametrize("shape,V,path", [([-1, 0, 0, 1, 1, 2, 2], 4, "auto"),
+                                          ([-1, 0, 0, 0, 1, 1, 2, 4], 3, "auto"),
+                                          ([-1, 0, 1, 2], 8, "persistent"),
+                                          ([-1, 0, 0, 1, 1, 2, 2], 8, "cluster")])
+def test_kernel_output_law_is_target(tv, shape, V, path):
+    """V = 3 and 4 take the three-kernel path (V % 8 != 0); V = 8 runs the
+    persistent kernel and the cluster kernel."""
+    obs, exp = z_counts(tv, shape, V, 1_000_000, seed=V * 17 + len(shape), path=path)
     assert chi2_p(obs, exp) > 1e-3
 
 
