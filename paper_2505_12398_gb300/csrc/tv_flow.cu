@@ -15,7 +15,9 @@
 //   * an owner warp runs the serial control of the CTA's current tree (tree
 //     set-up, combining partials, Eqs. (1)-(3), posting the next job);
 //   * a fetcher warp takes tickets and copies the queued slices into the
-//     CTA's slots, up to two slices ahead of the one being reduced;
+//     CTA's slots, one slice ahead of the one being reduced (a second slice
+//     held ahead made jobs wait longer behind other trees' slices: 3-5 %
+//     slower at 128 to 1024 trees);
 //   * a producer warp streams the fetched slices into a shared-memory ring
 //     with 1-D bulk copies (TMA);
 //   * NCW consumer warps reduce the ring stages and write each slice's
@@ -53,7 +55,7 @@ namespace flow {
 using namespace tvk::fused;
 
 constexpr int kMaxNCW = 8;
-constexpr int kSlots = 3;           // queued slices a CTA holds: one streaming, two ahead
+constexpr int kSlots = 2;           // queued slices a CTA holds: one streaming, one ahead
 constexpr int kPBuf = 256;          // partials of a job kept in shared memory by the poll
 constexpr unsigned long long kNoPart = ~0ull;   // a partial slot not written yet
 constexpr unsigned kNoTicket = 0xffffffffu;
