@@ -69,7 +69,6 @@ enum : int {
 };
 enum : int { kStageFirst = 1, kStageLast = 2, kStageExit = 4 };
 constexpr int kSlotExit = -1;       // ItemSlot::kind of the fetcher's "no more slices"
-constexpr int kItemNop = 6;         // FlowItem::kind of a reserved slot that carries no work
 
 // A queued slice as held by a CTA (the masks live in shared arrays of R).
 struct ItemSlot {
@@ -216,7 +215,7 @@ __device__ void fetcher_role(const TravArgs& a, const FlowArgs& f, const Smem& m
     }
     ItemSlot& it = m.sh->slots[slot];
     // ---- a ticket, then its slot's publication (lane 0) ----
-    int cmd = 0;   // 1: a slice, 2: stop, 3: a reserved slot without work
+    int cmd = 0;   // 1: a slice, 2: stop
     if (lane == 0) {
       unsigned ticket = kNoTicket;
       if (ld_relaxed_u32(&f.ctr[kCtrDone]) >= (unsigned)B) cmd = 2;   // nothing will come
@@ -242,7 +241,6 @@ __device__ void fetcher_role(const TravArgs& a, const FlowArgs& f, const Smem& m
         const int4* bp = reinterpret_cast<const int4*>(f.items + ticket);
 #pragma unroll
         for (int k = 0; k < 7; ++k) w[k] = __ldcg(bp + k);   // one 112-byte read
-        if (w[1].x == kItemNop) cmd = 3;
       }
       if (cmd == 1) {
         it.b = w[0].x; it.node = w[0].y; it.row = w[0].z; it.slice = w[0].w;
@@ -263,7 +261,6 @@ __device__ void fetcher_role(const TravArgs& a, const FlowArgs& f, const Smem& m
     }
     cmd = __shfl_sync(0xffffffffu, cmd, 0);
     __syncwarp();
-    if (cmd == 3) continue;   // keep the slot for the next ticket
     if (cmd == 1) {
       const int nmask = it.nmask;
       if (nmask > kFlowInlineMask) {   // rare: the rest of a long mask list
@@ -622,13 +619,6 @@ __device__ void consumer_role(const TravArgs& a, const FlowArgs& f, const Smem& 
 
 // --------------------------------------------------------------- owner --
 
-// Queue slots reserved ahead of the job that will use them (see owner_role).
-struct Reserve {
-  unsigned base;
-  int n;       // 0: none
-  int slice;
-};
-
 // Tokens per slice: enough slices per row to give every CTA one when each
 // remaining tree has a job out, between the plan's largest and smallest
 // slice.  Early on (many trees) this keeps slices large; towards the end,
@@ -644,51 +634,16 @@ __device__ __forceinline__ int adaptive_slice(const FlowArgs& f, int V, int B, b
   return max(f.slice_min, min(largest, want));
 }
 
-// Writes "no work" items into reserved slots [base, base + n) (before the
-// caller's fence) ...
-__device__ __forceinline__ void nop_bodies(const FlowArgs& f, unsigned base, int n, int lane) {
-  for (int q = lane; q < n; q += 32)
-    __stcg(reinterpret_cast<int4*>(f.items + base + q) + 1, make_int4(kItemNop, 0, 0, 0));
-}
-
-// ... and, after it, their tags.
-__device__ __forceinline__ void nop_tags(const FlowArgs& f, unsigned base, int n, int lane) {
-  for (int q = lane; q < n; q += 32)
-    st_relaxed_u64(&f.items[base + q].tag, (f.epoch << 32) | (unsigned long long)(base + q));
-}
-
-// Publishes reserved slots that no job will use.
-__device__ void post_nops(const TravArgs& a, const FlowArgs& f, Reserve spec, int lane) {
-  if ((size_t)spec.base + spec.n + kMaxGrid > (size_t)f.cap) {
-    if (lane == 0) raise_abort(a, f);
-    return;
-  }
-  nop_bodies(f, spec.base, spec.n, lane);
-  fence_gpu();
-  __syncwarp();
-  nop_tags(f, spec.base, spec.n, lane);
-}
-
-// Reserves the queue slots of a rejection pass of the current size (lane 0;
-// not after a bonus draw, which ends the tree).
-__device__ __forceinline__ void reserve_next(const FlowArgs& f, int V, int B, int posted_kind,
-                                             unsigned done, Reserve& spec) {
-  spec.n = 0;
-  if (posted_kind == kJobBonusLeaf || posted_kind == kJobBonusRes) return;
-  spec.slice = adaptive_slice(f, V, B, false, 1, done);
-  spec.n = (V + spec.slice - 1) / spec.slice;
-  spec.base = atomicAdd(&f.ctr[kCtrTail], (unsigned)spec.n);
-}
-
-// Publishes the own tree's current job (ctl.job) as slice items.  A pass may
-// use the slots reserved in `spec`; otherwise those become "no work" items.
+// Publishes the own tree's current job (ctl.job) as slice items.  (Its queue
+// slots are taken when the items are written: slots reserved earlier, to
+// overlap that atomic with the combine, held the fetchers that drew them
+// until the job was published, 1-1.5 % slower.)
 __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const FlowArgs& f,
-                         int b, int V, int lane, unsigned done, Reserve spec, const Job& j,
+                         int b, int V, int lane, unsigned done, const Job& j,
                          const int* mask_tok, const float* mask_val) {
   const bool stats = (j.kind == kJobStats);
   const int n_rows = stats ? j.n_rows : 1;
-  const bool use_spec = spec.n > 0 && j.kind == kJobPass;
-  const int slice = use_spec ? spec.slice : adaptive_slice(f, V, a.B, stats, n_rows, done);
+  const int slice = adaptive_slice(f, V, a.B, stats, n_rows, done);
   const int K = (V + slice - 1) / slice;
   const int nmask = (j.kind == kJobPass || j.kind == kJobBonusRes) ? j.nmask : 0;
   const int n = n_rows * K;
@@ -702,19 +657,15 @@ __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const
     const int r = q / K;
     __stcg(f.part + ((size_t)b * R + r) * f.Kmax + (q - r * K), kNoPart);
   }
-  unsigned base = spec.base;
-  if (!use_spec) {
-    if (lane == 0) base = atomicAdd(&f.ctr[kCtrTail], (unsigned)n);
-    base = __shfl_sync(0xffffffffu, base, 0);
-  }
+  unsigned base = 0u;
+  if (lane == 0) base = atomicAdd(&f.ctr[kCtrTail], (unsigned)n);
+  base = __shfl_sync(0xffffffffu, base, 0);
   // the last kMaxGrid slots are kept for exit tags; a correctly sized queue
   // never reaches them
-  if ((size_t)base + n + kMaxGrid > (size_t)f.cap ||
-      (spec.n > 0 && (size_t)spec.base + spec.n + kMaxGrid > (size_t)f.cap)) {
+  if ((size_t)base + n + kMaxGrid > (size_t)f.cap) {
     if (lane == 0) raise_abort(a, f);
     return;
   }
-  if (spec.n > 0 && !use_spec) nop_bodies(f, spec.base, spec.n, lane);
   const int4 w1 = make_int4(j.kind, slice, nmask, 0);
   const int4 w2 = make_int4(__float_as_int(j.alpha1), __float_as_int(j.beta),
                             __float_as_int(j.rowmax), 0);
@@ -751,7 +702,6 @@ __device__ void post_job(const TreeSmem& s, Shared& sh, const TravArgs& a, const
   if (b != f.withhold_tree)
     for (int q = lane; q < n; q += 32)
       st_relaxed_u64(&f.items[base + q].tag, (f.epoch << 32) | (unsigned long long)(base + q));
-  if (spec.n > 0 && !use_spec) nop_tags(f, spec.base, spec.n, lane);
   if (lane == 0) {
     sh.outstanding = n;
     sh.jkind = j.kind;
@@ -1155,7 +1105,6 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
   unsigned polls = 0u;
   Backoff wait;
   unsigned done_est = 0u;      // trees finished, as read after the last post
-  Reserve spec{0u, 0, 0};      // slots reserved for the next job (lane 0's copy counts)
   for (;;) {
     __syncwarp();   // lane 0's updates of sh (job shape, control state) seen by all lanes
     if (my_tree < 0) {
@@ -1193,11 +1142,6 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
         continue;
       }
       wait.reset();
-      // after a pass the next job is most often a pass of the same row size:
-      // reserve its queue slots now, so that the reservation's round trip
-      // overlaps the combine.  (Reserving earlier, while the job runs, holds
-      // fetchers on slots that stay unpublished for microseconds.)
-      if (lane == 0 && sh.jkind == kJobPass) reserve_next(f, V, B, kJobPass, done_est, spec);
       // the bonus draw reads tiles written before its partials
       if (sh.jkind == kJobBonusLeaf || sh.jkind == kJobBonusRes) fence_gpu();
       __syncwarp();
@@ -1250,21 +1194,17 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
         if (fast) {
           post_first = __shfl_sync(0xffffffffu, post_first, 0);
           accept = __shfl_sync(0xffffffffu, accept, 0);
-          spec.base = __shfl_sync(0xffffffffu, spec.base, 0);
-          spec.n = __shfl_sync(0xffffffffu, spec.n, 0);
-          spec.slice = __shfl_sync(0xffffffffu, spec.slice, 0);
           __syncwarp();
           if (post_first) {
             post_job(s, sh, a, f, my_tree, V, lane, __shfl_sync(0xffffffffu, done_est, 0),
-                     spec, sh.fjob, m.mtok2, s.mask_val);
+                     sh.fjob, m.mtok2, s.mask_val);
             if (lane == 0) control_step_ahead(s, sh.ctl, sh.ahead, accept != 0);
           } else {
             if (lane == 0) control_step_ahead(s, sh.ctl, sh.ahead, accept != 0);
             __syncwarp();
             post_job(s, sh, a, f, my_tree, V, lane, __shfl_sync(0xffffffffu, done_est, 0),
-                     spec, sh.ctl.job, s.mask_tok, s.mask_val);
+                     sh.ctl.job, s.mask_tok, s.mask_val);
           }
-          spec.n = 0;
           if (lane == 0) {
             done_est = ld_relaxed_u32(&f.ctr[kCtrDone]);
             if (a.token_level) sh.ahead.ok = 0;            // (Traversal Verification only)
@@ -1275,12 +1215,7 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
       }
       owner_combine<L>(a, f, s, sh, m.u, my_tree, lane);
     }
-    spec.base = __shfl_sync(0xffffffffu, spec.base, 0);
-    spec.n = __shfl_sync(0xffffffffu, spec.n, 0);
-    spec.slice = __shfl_sync(0xffffffffu, spec.slice, 0);
     if (sh.ctl.job.kind == kJobDone) {
-      if (spec.n > 0) post_nops(a, f, spec, lane);   // before the tree counts as done
-      spec.n = 0;
       const bool last = owner_finish<kGiven>(a, f, s, sh, m.u, my_tree, lane);
       my_tree = -1;
       if (last) {
@@ -1298,9 +1233,8 @@ __device__ void owner_role(const TravArgs& a, const FlowArgs& f, const Smem& m, 
           st_relaxed_u64(&f.items[q].tag, (f.epoch << 32) | q | kExitTag);
       }
     } else {
-      post_job(s, sh, a, f, my_tree, V, lane, __shfl_sync(0xffffffffu, done_est, 0), spec,
+      post_job(s, sh, a, f, my_tree, V, lane, __shfl_sync(0xffffffffu, done_est, 0),
                sh.ctl.job, s.mask_tok, s.mask_val);
-      spec.n = 0;
       if (lane == 0) {
         done_est = ld_relaxed_u32(&f.ctr[kCtrDone]);   // used at the next job
         if (a.token_level) sh.ahead.ok = 0;             // (Traversal Verification only)
@@ -1399,8 +1333,8 @@ FlowLayout flow_layout(int B, int R, int V, int min_slice) {
   FlowLayout l;
   l.kmax = (size_t)((V + min_slice - 1) / min_slice);
   // per tree: at most R rows normalised and at most R - 1 passes plus the
-  // bonus draw, each at most kmax slices, and for each job at most one range
-  // reserved ahead and left unused; then room for the exit tags
+  // bonus draw, each at most kmax slices, with a factor of two to spare; then
+  // room for the exit tags
   l.cap = (size_t)B * (4 * (size_t)R + 2) * l.kmax + tvk::flow::kMaxGrid;
   l.ntiles = (size_t)((V + tvk::fused::kTileElems - 1) / tvk::fused::kTileElems);
   return l;
