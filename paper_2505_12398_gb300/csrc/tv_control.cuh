@@ -16,9 +16,10 @@
 namespace tvk {
 namespace fused {
 
-// A CTA has NCW consumer warps (4 or 8) and one producer warp; its ring
-// stages hold 3 * NCW KB: a target + draft slice of 512 * NCW tokens (bf16),
-// or a target-only slice of 1536 * NCW tokens.
+// A CTA of the cluster kernel has NCW consumer warps (4 or 8) and one producer
+// warp; its ring stages hold 3 * NCW KB: a target + draft slice of 512 * NCW
+// tokens (bf16), or a target-only slice of 1536 * NCW tokens.  (The
+// persistent kernel sizes its stages itself, tv_flow.cu.)
 constexpr int kMaxStages = 8;
 constexpr int kMaxCluster = 8;
 constexpr int kTileElems = 256;       // one warp x 8 elements

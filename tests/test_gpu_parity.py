@@ -135,6 +135,23 @@ def test_fused_launch_shapes(tv, shape, monkeypatch):
     check(tv, inp, path="cluster")
 
 
+@pytest.mark.parametrize("plan", ["4,2,0,0,0", "4,3,0,0,0", "8,2,0,0,0", "4,0,4096,8192,2048"])
+def test_persistent_launch_shapes(tv, plan, monkeypatch):
+    """Other launch shapes of the persistent kernel (TV_FLOW_PLAN: consumer
+    warps, ring stages, pass / normaliser / smallest slice tokens) give the
+    oracle's results: three 18 KB stages (three CTAs per SM), eight consumer
+    warps, and slices small enough for several per row (V=32000, EAGLE trees)."""
+    monkeypatch.setenv("TV_FLOW_PLAN", plan)
+    w = get_workload("eagle_v32k", batch=24)
+    inp = make_inputs(w, seed=25, device="cuda")
+    v = tv.Verifier(w.vocab, w.nodes, 24, "bf16", path="persistent")
+    path, _, warps, stages = v.launch_shape(24, w.nodes)
+    v.close()
+    ncw, st = (int(x) for x in plan.split(",")[:2])
+    assert path == 2 and warps == ncw and (st == 0 or stages == st)
+    check(tv, inp, path="persistent")
+
+
 @pytest.mark.parametrize("batch", [1, 8, 40, 400, 1000])
 @pytest.mark.parametrize("path", ["persistent", "cluster"])
 def test_default_launch_shapes(tv, batch, path):
