@@ -1402,14 +1402,19 @@ FlowPlan tv_flow_plan(int R, int B, int V, int smem_per_sm, int smem_per_block, 
   // token slices stream 14 % faster than 8192; at 128 trees, where a job's
   // latency sets the time, 8192 is best).  From 1024 trees a pass takes a
   // quarter row per slice and a normaliser half a row when that is larger
-  // (V = 151936: 38144 and 76032 tokens, 4 % faster than 32768 for both; V =
-  // 128256: 64256-token normaliser slices, 4 % faster)
-  auto tiles_up = [](long long x) { return (int)((x + 255) / 256 * 256); };
-  p.slice_pass = B >= 1024 ? std::max(32768, tiles_up((V + 3LL) / 4))
-                           : (B >= 256 ? 16384 : 8192);
-  p.slice_stats = B >= 1024 ? std::max(32768, tiles_up((V + 1LL) / 2))
-                            : (B >= 256 ? 32768 : 16384);
+  // (V = 151936: 4 % faster than 32768 for both; V = 128256: 64512-token
+  // normaliser slices, 4 % faster), rounded up to whole ring stages of bf16
+  // rows (3072 tokens of a pass, 9216 of a normaliser with four consumer
+  // warps; V = 151936: 39936 and 82944 tokens, 0.8 % faster than 38144 and
+  // 76032, whose last stages were partly empty)
   if (force_ncw == 4 || force_ncw == 8) p.ncw = force_ncw;
+  const long long pass_unit = tvk::flow::flow_stage_bytes(p.ncw) / 6 / 256 * 256;
+  const long long row_unit = tvk::flow::flow_stage_bytes(p.ncw) / 2;
+  auto up_to = [](long long x, long long unit) { return (int)((x + unit - 1) / unit * unit); };
+  p.slice_pass = B >= 1024 ? std::max(32768, up_to((V + 3LL) / 4, pass_unit))
+                           : (B >= 256 ? 16384 : 8192);
+  p.slice_stats = B >= 1024 ? std::max(32768, up_to((V + 1LL) / 2, row_unit))
+                            : (B >= 256 ? 32768 : 16384);
   if (force_slice_pass >= 256 && force_slice_pass % 256 == 0) p.slice_pass = force_slice_pass;
   if (force_slice_stats >= 256 && force_slice_stats % 256 == 0) p.slice_stats = force_slice_stats;
   if (force_slice_min >= 256 && force_slice_min % 256 == 0) p.slice_min = force_slice_min;
