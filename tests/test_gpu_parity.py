@@ -152,6 +152,18 @@ def test_persistent_launch_shapes(tv, plan, monkeypatch):
     check(tv, inp, path="persistent")
 
 
+@pytest.mark.parametrize("V,N,want", [(32000, 60, 1), (49152, 127, 1), (32000, 200, 2),
+                                       (50000, 60, 2), (128256, 60, 2), (1003, 60, 0)])
+def test_auto_path_choice(tv, V, N, want):
+    """A handle that picks its path itself: the cluster kernel for short rows
+    (V <= 49152, N + 1 <= 128), the persistent kernel otherwise, the
+    three-kernel path when V % 8 != 0 (tv_launch_shape's path codes 1, 2, 0)."""
+    v = tv.Verifier(V, N, 64, "bf16")
+    path, _, _, _ = v.launch_shape(64, N)
+    v.close()
+    assert path == want
+
+
 @pytest.mark.parametrize("batch", [1, 8, 40, 400, 1000])
 @pytest.mark.parametrize("path", ["persistent", "cluster"])
 def test_default_launch_shapes(tv, batch, path):
